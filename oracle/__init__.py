@@ -1,0 +1,125 @@
+"""fp64 CPU oracle for softmax attention forward (ctypes wrapper of oracle.c).
+
+TEST INFRASTRUCTURE ONLY: the tests, ``__graft_entry__.smoke()`` and the
+bench's ``cpu_baseline`` / ``--impl reference`` legs are the only callers.
+The product path (``paper_2609_18077_gb300``) never imports this package,
+and this package imports nothing from it.
+
+What the oracle computes is the plain softmax-attention definition (vidax
+paper, Sec. 2 "3D RoPE, 3D VAEs, and flash attention": flash attention is
+an exact re-ordering of it), with padded text keys excluded per sample
+(appendix Table 4, segment-id masking of invalid key blocks).  See the
+header of ``oracle.c`` for the formulas.
+
+Inputs are bf16 bit patterns as ``numpy.uint16`` arrays ``[B, H, S, D]``;
+outputs are ``float64``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+SOURCE = os.path.join(_HERE, "oracle.c")
+LIBRARY = os.path.join(_HERE, "liboracle.so")
+
+
+def build(source: str = SOURCE, output: str = LIBRARY, extra_flags=()) -> str:
+    """Compile ``oracle.c`` with gcc (fp64, OpenMP, no fast-math)."""
+    cmd = ["gcc", "-O2", "-fopenmp", "-shared", "-fPIC", "-std=c99",
+           *extra_flags, "-o", output, source, "-lm"]
+    subprocess.run(cmd, check=True, capture_output=True, text=True)
+    return output
+
+
+class Oracle:
+    """Handle on one compiled oracle library (the real one, or a test mutant)."""
+
+    def __init__(self, path: str = LIBRARY):
+        if not os.path.exists(path):
+            raise FileNotFoundError(f"oracle library {path} is not built; call oracle.build()")
+        self.path = path
+        lib = ctypes.CDLL(path)
+        lib.oracle_attn_fwd.restype = ctypes.c_int
+        lib.oracle_attn_fwd.argtypes = [
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+            ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
+        lib.oracle_set_threads.restype = ctypes.c_int
+        lib.oracle_set_threads.argtypes = [ctypes.c_int]
+        self._lib = lib
+
+    def set_threads(self, n: int = 0) -> int:
+        """Set the OpenMP thread count (n <= 0 keeps it); returns the count in use."""
+        return int(self._lib.oracle_set_threads(int(n)))
+
+    def attn_fwd(self, q, k, v, scale, kv_lens=None, rows=None, probs=False):
+        """Attention forward in fp64.
+
+        q: uint16 [B,H,Sq,D]; k, v: uint16 [B,H,Skv,D] (bf16 bits).
+        kv_lens: None or int [B] (valid keys per sample, clamped to [0, Skv]).
+        rows: None (all query rows) or int [B*H, n] query indices per (b, h).
+        Returns (o [B,H,n,D] f64, lse [B,H,n] f64[, probs [B,H,n,Skv] f64]).
+        """
+        q = _bits(q)
+        k = _bits(k)
+        v = _bits(v)
+        B, H, Sq, D = q.shape
+        Skv = k.shape[2]
+        if k.shape != (B, H, Skv, D) or v.shape != (B, H, Skv, D):
+            raise ValueError("k and v must be [B,H,Skv,D] matching q")
+        lens = None
+        if kv_lens is not None:
+            lens = np.ascontiguousarray(np.asarray(kv_lens, dtype=np.int32))
+            if lens.shape != (B,):
+                raise ValueError("kv_lens must have shape [B]")
+        if rows is None:
+            n = Sq
+            rows_arr = None
+        else:
+            rows_arr = np.ascontiguousarray(np.asarray(rows, dtype=np.int32))
+            if rows_arr.ndim != 2 or rows_arr.shape[0] != B * H:
+                raise ValueError("rows must have shape [B*H, n]")
+            n = rows_arr.shape[1]
+        o = np.empty((B, H, n, D), dtype=np.float64)
+        lse = np.empty((B, H, n), dtype=np.float64)
+        pr = np.empty((B, H, n, Skv), dtype=np.float64) if probs else None
+        rc = self._lib.oracle_attn_fwd(
+            _ptr(q), _ptr(k), _ptr(v), B, H, Sq, Skv, D, float(scale),
+            _ptr(lens), _ptr(rows_arr), n, _ptr(o), _ptr(lse), _ptr(pr))
+        if rc != 0:
+            raise RuntimeError("oracle_attn_fwd rejected its arguments")
+        return (o, lse, pr) if probs else (o, lse)
+
+
+def _bits(a) -> np.ndarray:
+    a = np.asarray(a)
+    if a.dtype != np.uint16 or a.ndim != 4:
+        raise TypeError("oracle inputs are uint16 bf16 bit patterns of rank 4")
+    return np.ascontiguousarray(a)
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+_default = None
+
+
+def default() -> Oracle:
+    """The oracle built from ``oracle.c`` (compiled on first use if missing)."""
+    global _default
+    if _default is None:
+        if not os.path.exists(LIBRARY) or os.path.getmtime(LIBRARY) < os.path.getmtime(SOURCE):
+            build()
+        _default = Oracle(LIBRARY)
+    return _default
+
+
+def attn_fwd(q, k, v, scale, kv_lens=None, rows=None, probs=False):
+    """Module-level shortcut for ``default().attn_fwd``."""
+    return default().attn_fwd(q, k, v, scale, kv_lens=kv_lens, rows=rows, probs=probs)

@@ -1,0 +1,185 @@
+"""Seeded synthetic attention workloads shaped like the paper's video DiTs.
+
+This module only draws inputs; it holds none of the attention arithmetic and
+is the one piece shared by the CUDA path's tests and the CPU oracle.
+
+Geometry: a latent video of F x Hp x Wp patches flattened to S = F*Hp*Wp
+tokens per sample (vidax paper, Sec. 1: patchifying temporal volumes gives
+sequences of tens of thousands of tokens; the Wan2.1 832x480 and 1280x720,
+81-frame rows of Table 5 give 21x30x52 and 21x45x80 latents).  Cross-attention
+attends video tokens to a padded batch of text tokens with per-sample valid
+lengths (Sec. 3.1, Wan's UMT5 text conditioning; appendix Table 4 on masking
+padded text tokens).  Classifier-free guidance doubles the internal batch
+(Sec. 4, experimental setup), hence B = 2 for the text cross-attention.
+
+Recipe (every draw is seeded; no dataset is read):
+  * rng = numpy PCG64(seed); Q, K, V ~ N(0, 1) float32, drawn in that order;
+  * "logit std ~ 3": Q and K are multiplied by sqrt(3) in float32 before the
+    bf16 cast, so with scale = 1/sqrt(D) the logits scale*q.k have std ~ 3;
+  * cast to bf16 by round-to-nearest-even (torch CPU);
+  * outlier keys: per sample, round(frac * Skv) token positions drawn without
+    replacement (shared by all heads), those K rows multiplied by 8 after the
+    cast (exact: a power of two);
+  * text lengths: one integer per sample, uniform on the inclusive range
+    [lo, hi]; K/V rows past a sample's length are padding and may be filled
+    with NaN to prove they are never read;
+  * row subsets for large configs: per (b, h), n distinct query rows.
+Independent streams (lengths, outliers, row subsets) come from
+SeedSequence(seed).spawn so that adding one never shifts another.
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field
+
+import numpy as np
+import torch
+
+BF16_NAN_BITS = 0x7FC0
+
+
+@dataclass(frozen=True)
+class Workload:
+    """One attention problem: shapes plus the recipe of its synthetic inputs."""
+    name: str
+    B: int
+    H: int
+    D: int
+    Sq: int
+    Skv: int
+    seed: int
+    latent: tuple = ()            # (frames, rows, cols) of patches, when Sq comes from one
+    logit_gain: float = 1.0       # Q and K are scaled by this before the bf16 cast
+    outlier_frac: float = 0.0     # fraction of K rows multiplied by 8
+    kv_len_range: tuple | None = None   # inclusive (lo, hi) per-sample text lengths
+    oracle_rows: int | None = None      # per (b, h) query rows the parity check compares
+    description: str = field(default="", compare=False)
+
+    @property
+    def scale(self) -> float:
+        return 1.0 / math.sqrt(self.D)
+
+    @property
+    def varlen(self) -> bool:
+        return self.kv_len_range is not None
+
+    def flops(self, kv_lens=None) -> float:
+        """Algorithmic FLOPs 4*B*H*Sq*Skv*D (two GEMMs, 2 flops per MAC).
+
+        With kv_lens the effective count uses the valid keys of each sample.
+        """
+        if kv_lens is None:
+            return 4.0 * self.B * self.H * self.Sq * self.Skv * self.D
+        return 4.0 * self.H * self.Sq * self.D * float(np.sum(np.clip(kv_lens, 0, self.Skv)))
+
+
+WORKLOADS = {
+    "tiny": Workload(
+        "tiny", B=1, H=2, D=64, Sq=192, Skv=192, seed=1001, latent=(3, 8, 8),
+        description="tiny self-attention, latent 3x8x8 -> 192 tokens"),
+    "small480": Workload(
+        "small480", B=1, H=12, D=128, Sq=32760, Skv=32760, seed=1002, latent=(21, 30, 52),
+        logit_gain=math.sqrt(3.0), oracle_rows=4096,
+        description="small-DiT 480p self-attention, latent 21x30x52 -> 32760 tokens, logit std ~3"),
+    "cross": Workload(
+        "cross", B=2, H=12, D=128, Sq=32760, Skv=512, seed=1003, latent=(21, 30, 52),
+        kv_len_range=(64, 512),
+        description="video-to-text cross-attention, 32760 video tokens x <=512 text tokens, CFG batch 2"),
+    "large480": Workload(
+        "large480", B=1, H=40, D=128, Sq=32760, Skv=32760, seed=1004, latent=(21, 30, 52),
+        logit_gain=math.sqrt(3.0), outlier_frac=0.05, oracle_rows=4096,
+        description="large-DiT 480p self-attention, logit std ~3, 5% outlier key rows x8"),
+    "large720": Workload(
+        "large720", B=1, H=40, D=128, Sq=75600, Skv=75600, seed=1005, latent=(21, 45, 80),
+        oracle_rows=4096,
+        description="large-DiT 720p self-attention, latent 21x45x80 -> 75600 tokens"),
+}
+
+# The bench's default workload: the small-DiT 480p self-attention.
+DEFAULT_WORKLOAD = "small480"
+
+
+def _spawn(seed: int, n: int = 3):
+    return [np.random.Generator(np.random.PCG64(s)) for s in np.random.SeedSequence(seed).spawn(n)]
+
+
+def to_bf16(a: np.ndarray) -> torch.Tensor:
+    """float32 numpy -> bf16 torch CPU tensor (round to nearest even)."""
+    return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16)
+
+
+def bf16_bits(t: torch.Tensor) -> np.ndarray:
+    """bf16 torch tensor -> numpy uint16 bit patterns (same shape, CPU copy)."""
+    return t.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+
+
+def random_qkv(B, H, Sq, Skv, D, seed, logit_gain=1.0):
+    """Q, K, V as bf16 CPU tensors, N(0,1) with Q and K scaled by logit_gain."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    q = rng.standard_normal((B, H, Sq, D), dtype=np.float32)
+    k = rng.standard_normal((B, H, Skv, D), dtype=np.float32)
+    v = rng.standard_normal((B, H, Skv, D), dtype=np.float32)
+    if logit_gain != 1.0:
+        g = np.float32(logit_gain)
+        q *= g
+        k *= g
+    return to_bf16(q), to_bf16(k), to_bf16(v)
+
+
+def draw_kv_lens(B, lo, hi, seed) -> np.ndarray:
+    """Per-sample valid key counts, uniform on the inclusive range [lo, hi]."""
+    rng = _spawn(seed)[0]
+    return rng.integers(lo, hi + 1, size=B, dtype=np.int64).astype(np.int32)
+
+
+def draw_outlier_rows(B, Skv, frac, seed) -> list:
+    """Per sample, round(frac*Skv) distinct key positions (sorted)."""
+    rng = _spawn(seed)[1]
+    n = int(round(frac * Skv))
+    return [np.sort(rng.choice(Skv, size=n, replace=False)) for _ in range(B)]
+
+
+def draw_rows(B, H, Sq, n, seed) -> np.ndarray:
+    """Per (b, h), n distinct query rows (sorted), shape [B*H, n] int32."""
+    rng = _spawn(seed)[2]
+    n = min(n, Sq)
+    return np.stack([np.sort(rng.choice(Sq, size=n, replace=False)) for _ in range(B * H)]).astype(np.int32)
+
+
+def pad_invalid_keys(k: torch.Tensor, v: torch.Tensor, kv_lens, fill_bits: int = BF16_NAN_BITS):
+    """Overwrite K/V rows past each sample's valid length with a bf16 bit pattern."""
+    k = k.clone()
+    v = v.clone()
+    kb = k.view(torch.int16)
+    vb = v.view(torch.int16)
+    fill = np.array(fill_bits, dtype=np.uint16).view(np.int16).item()
+    for b, L in enumerate(np.asarray(kv_lens)):
+        L = int(max(0, min(int(L), k.shape[2])))
+        kb[b, :, L:, :] = fill
+        vb[b, :, L:, :] = fill
+    return k, v
+
+
+def generate(w: Workload | str, nan_padding: bool = True):
+    """Materialise a workload on the CPU.
+
+    Returns a dict with q, k, v (bf16 CPU tensors [B,H,S,D]), scale,
+    kv_lens (int32 numpy [B] or None), rows (int32 [B*H, n] or None: the
+    query rows a parity check compares) and the workload itself.
+    """
+    if isinstance(w, str):
+        w = WORKLOADS[w]
+    q, k, v = random_qkv(w.B, w.H, w.Sq, w.Skv, w.D, w.seed, w.logit_gain)
+    if w.outlier_frac > 0:
+        for b, idx in enumerate(draw_outlier_rows(w.B, w.Skv, w.outlier_frac, w.seed)):
+            k[b, :, torch.from_numpy(idx.astype(np.int64)), :] *= 8
+    kv_lens = None
+    if w.kv_len_range is not None:
+        kv_lens = draw_kv_lens(w.B, w.kv_len_range[0], w.kv_len_range[1], w.seed)
+        if nan_padding:
+            k, v = pad_invalid_keys(k, v, kv_lens)
+    rows = None
+    if w.oracle_rows is not None and w.oracle_rows < w.Sq:
+        rows = draw_rows(w.B, w.H, w.Sq, w.oracle_rows, w.seed)
+    return {"workload": w, "q": q, "k": k, "v": v, "scale": w.scale,
+            "kv_lens": kv_lens, "rows": rows}

@@ -1,0 +1,232 @@
+"""Pins of the fp64 oracle to facts other than itself.
+
+Each pin takes an ``oracle.Oracle`` handle and raises AssertionError when the
+oracle disagrees with a closed form, an invariant of softmax attention, an
+independent library routine or a high-precision brute-force evaluation.
+``test_oracle.py`` runs them on the real oracle; ``test_oracle_mutants.py``
+runs them on copies of the oracle with planted mistakes and requires every
+mistake to be caught by at least one pin.
+
+Sources of the facts (none of them is the oracle's own code):
+  * closed forms of softmax attention with one or two keys;
+  * invariants: weights sum to one, constant values are returned unchanged,
+    query-row permutation equivariance, joint key/value permutation
+    invariance, translation of values, zero logits give the mean;
+  * masking: a sample with L valid keys equals dense attention on the first
+    L keys, whatever the padding holds (appendix Table 4 of the paper:
+    padded text tokens must not be attended);
+  * torch's scaled_dot_product_attention and logsumexp in fp64 (a library);
+  * a 50-digit mpmath evaluation on a tiny input.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+from paper_2609_18077_gb300.workloads import bf16_bits, random_qkv, to_bf16, pad_invalid_keys
+
+TOL = 1e-12
+
+
+def _dec(bits) -> np.ndarray:
+    """bf16 bit patterns -> float64 (exact), independent of the oracle."""
+    return (np.asarray(bits, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def _bits_of(values) -> np.ndarray:
+    return bf16_bits(to_bf16(np.asarray(values, dtype=np.float32)))
+
+
+def _inputs(B, H, Sq, Skv, D, seed, gain=1.0):
+    q, k, v = random_qkv(B, H, Sq, Skv, D, seed, gain)
+    return bf16_bits(q), bf16_bits(k), bf16_bits(v)
+
+
+def pin_single_key(orc):
+    """Skv = 1: o = v_0 exactly and lse = scale * q.k_0."""
+    q, k, v = _inputs(2, 3, 5, 1, 16, seed=11)
+    scale = 0.37
+    o, lse = orc.attn_fwd(q, k, v, scale)
+    qd, kd, vd = _dec(q), _dec(k), _dec(v)
+    np.testing.assert_allclose(o, np.broadcast_to(vd, o.shape), rtol=0, atol=TOL)
+    want = scale * np.einsum("bhid,bhjd->bhi", qd, kd)
+    np.testing.assert_allclose(lse, want, rtol=TOL, atol=TOL)
+
+
+def pin_two_keys(orc):
+    """Skv = 2: o = (1-w) v_0 + w v_1 with w = sigmoid(s_1 - s_0); lse = log(e^s0 + e^s1)."""
+    q, k, v = _inputs(1, 2, 7, 2, 8, seed=12)
+    scale = 0.8
+    o, lse = orc.attn_fwd(q, k, v, scale)
+    qd, kd, vd = _dec(q), _dec(k), _dec(v)
+    s = scale * np.einsum("bhid,bhjd->bhij", qd, kd)
+    w = 1.0 / (1.0 + np.exp(s[..., 0] - s[..., 1]))
+    want_o = (1 - w)[..., None] * vd[:, :, 0:1, :] + w[..., None] * vd[:, :, 1:2, :]
+    np.testing.assert_allclose(o, want_o, rtol=0, atol=1e-12)
+    hi = np.maximum(s[..., 0], s[..., 1])
+    want_lse = hi + np.log1p(np.exp(-np.abs(s[..., 0] - s[..., 1])))
+    np.testing.assert_allclose(lse, want_lse, rtol=TOL, atol=TOL)
+
+
+def pin_weights_sum_to_one(orc):
+    """Softmax weights are non-negative and every row sums to one; o = P @ V."""
+    q, k, v = _inputs(2, 2, 9, 13, 16, seed=13, gain=2.0)
+    o, lse, p = orc.attn_fwd(q, k, v, 0.25, probs=True)
+    assert np.all(p >= 0)
+    np.testing.assert_allclose(p.sum(-1), 1.0, rtol=0, atol=1e-13)
+    np.testing.assert_allclose(o, p @ _dec(v), rtol=0, atol=1e-12)
+
+
+def pin_constant_values(orc):
+    """If every value row is the same vector c, the output is c."""
+    q, k, _ = _inputs(1, 2, 6, 11, 8, seed=14, gain=3.0)
+    c = np.array([1.5, -2.0, 0.25, 3.0, -0.125, 7.0, 0.0, -1.0], dtype=np.float32)
+    v = _bits_of(np.broadcast_to(c, (1, 2, 11, 8)))
+    o, _ = orc.attn_fwd(q, k, v, 0.5)
+    np.testing.assert_allclose(o, np.broadcast_to(c.astype(np.float64), o.shape), rtol=0, atol=1e-12)
+
+
+def pin_zero_logits(orc):
+    """scale = 0 (or q = 0): every weight is 1/L, o = mean of the L values, lse = ln L."""
+    q, k, v = _inputs(2, 2, 4, 10, 8, seed=15)
+    for case in ("scale", "q"):
+        if case == "scale":
+            o, lse = orc.attn_fwd(q, k, v, 0.0)
+        else:
+            o, lse = orc.attn_fwd(np.zeros_like(q), k, v, 0.9)
+        want = _dec(v).mean(axis=2, keepdims=True)
+        np.testing.assert_allclose(o, np.broadcast_to(want, o.shape), rtol=0, atol=1e-13)
+        np.testing.assert_allclose(lse, math.log(10), rtol=0, atol=1e-13)
+
+
+def pin_query_permutation(orc):
+    """Permuting query rows permutes o and lse the same way."""
+    q, k, v = _inputs(1, 2, 12, 9, 16, seed=16, gain=1.5)
+    perm = np.random.default_rng(1).permutation(12)
+    o, lse = orc.attn_fwd(q, k, v, 0.3)
+    o2, lse2 = orc.attn_fwd(np.ascontiguousarray(q[:, :, perm]), k, v, 0.3)
+    np.testing.assert_array_equal(o2, o[:, :, perm])
+    np.testing.assert_array_equal(lse2, lse[:, :, perm])
+
+
+def pin_key_value_permutation(orc):
+    """Permuting key rows and value rows jointly changes nothing (up to rounding)."""
+    q, k, v = _inputs(2, 1, 5, 17, 8, seed=17, gain=1.5)
+    perm = np.random.default_rng(2).permutation(17)
+    o, lse = orc.attn_fwd(q, k, v, 0.4)
+    o2, lse2 = orc.attn_fwd(q, np.ascontiguousarray(k[:, :, perm]), np.ascontiguousarray(v[:, :, perm]), 0.4)
+    np.testing.assert_allclose(o2, o, rtol=0, atol=1e-13)
+    np.testing.assert_allclose(lse2, lse, rtol=1e-14, atol=1e-13)
+
+
+def pin_value_translation(orc):
+    """Adding a constant row c to every value adds c to the output (weights sum to one)."""
+    # small integers keep v + c exactly representable in bf16
+    rng = np.random.default_rng(3)
+    q, k, _ = _inputs(1, 2, 5, 7, 4, seed=18)
+    vi = rng.integers(-8, 9, size=(1, 2, 7, 4)).astype(np.float32)
+    c = np.array([3.0, -5.0, 1.0, 16.0], dtype=np.float32)
+    o1, _ = orc.attn_fwd(q, k, _bits_of(vi), 0.6)
+    o2, _ = orc.attn_fwd(q, k, _bits_of(vi + c), 0.6)
+    np.testing.assert_allclose(o2 - o1, np.broadcast_to(c.astype(np.float64), o1.shape), rtol=0, atol=1e-12)
+
+
+def pin_varlen_is_truncation(orc):
+    """L valid keys (NaN padding after them) equal dense attention over the first L keys."""
+    B, H, Sq, Skv, D = 3, 2, 6, 20, 8
+    q, k, v = random_qkv(B, H, Sq, Skv, D, seed=19, logit_gain=1.2)
+    lens = np.array([20, 7, 1], dtype=np.int32)
+    kp, vp = pad_invalid_keys(k, v, lens)
+    o, lse = orc.attn_fwd(bf16_bits(q), bf16_bits(kp), bf16_bits(vp), 0.35, kv_lens=lens)
+    assert np.all(np.isfinite(o))
+    for b, L in enumerate(lens):
+        ob, lb = orc.attn_fwd(bf16_bits(q[b:b + 1]), bf16_bits(k[b:b + 1, :, :L]),
+                              bf16_bits(v[b:b + 1, :, :L]), 0.35)
+        np.testing.assert_array_equal(o[b:b + 1], ob)
+        np.testing.assert_array_equal(lse[b:b + 1], lb)
+
+
+def pin_varlen_empty_and_clamped(orc):
+    """L = 0 gives o = 0, lse = -inf; lengths beyond Skv clamp to Skv; negative to 0."""
+    q, k, v = _inputs(3, 1, 4, 5, 8, seed=20)
+    o, lse = orc.attn_fwd(q, k, v, 0.5, kv_lens=[0, 99, -3])
+    assert np.all(o[0] == 0) and np.all(np.isneginf(lse[0]))
+    assert np.all(o[2] == 0) and np.all(np.isneginf(lse[2]))
+    od, ld = orc.attn_fwd(q[1:2], k[1:2], v[1:2], 0.5)
+    np.testing.assert_array_equal(o[1:2], od)
+    np.testing.assert_array_equal(lse[1:2], ld)
+
+
+def pin_row_subset(orc):
+    """A row subset returns exactly the full result at those rows, per (b, h)."""
+    q, k, v = _inputs(2, 2, 11, 9, 8, seed=21)
+    rows = np.array([[10, 0, 3], [1, 2, 9], [5, 5, 7], [0, 10, 4]], dtype=np.int32)
+    o, lse = orc.attn_fwd(q, k, v, 0.7)
+    os_, ls = orc.attn_fwd(q, k, v, 0.7, rows=rows)
+    of = o.reshape(4, 11, 8)
+    lf = lse.reshape(4, 11)
+    for bh in range(4):
+        np.testing.assert_array_equal(os_.reshape(4, 3, 8)[bh], of[bh, rows[bh]])
+        np.testing.assert_array_equal(ls.reshape(4, 3)[bh], lf[bh, rows[bh]])
+
+
+def pin_torch_sdpa(orc):
+    """torch scaled_dot_product_attention and logsumexp in fp64 on the CPU (a library)."""
+    for (B, H, Sq, Skv, D, scale, seed) in [(1, 2, 17, 33, 64, 0.125, 22),
+                                             (2, 3, 40, 9, 128, 0.2, 23),
+                                             (1, 1, 5, 64, 16, -0.3, 24)]:
+        q, k, v = random_qkv(B, H, Sq, Skv, D, seed, logit_gain=1.7)
+        o, lse = orc.attn_fwd(bf16_bits(q), bf16_bits(k), bf16_bits(v), scale)
+        qd, kd, vd = q.double(), k.double(), v.double()
+        want = torch.nn.functional.scaled_dot_product_attention(qd, kd, vd, scale=scale)
+        want_lse = torch.logsumexp(scale * (qd @ kd.transpose(-1, -2)), dim=-1)
+        np.testing.assert_allclose(o, want.numpy(), rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse, want_lse.numpy(), rtol=1e-13, atol=1e-12)
+
+
+def pin_mpmath_brute_force(orc):
+    """A 50-digit evaluation of the definition on a 1x1x3x4 problem with 4 keys."""
+    import mpmath
+    mpmath.mp.dps = 50
+    q, k, v = _inputs(1, 1, 3, 4, 4, seed=25, gain=2.5)
+    scale = 0.45
+    o, lse = orc.attn_fwd(q, k, v, scale)
+    qd, kd, vd = _dec(q)[0, 0], _dec(k)[0, 0], _dec(v)[0, 0]
+    for i in range(3):
+        s = [mpmath.mpf(scale) * mpmath.fsum(mpmath.mpf(qd[i, d]) * mpmath.mpf(kd[j, d]) for d in range(4))
+             for j in range(4)]
+        e = [mpmath.e ** sj for sj in s]
+        z = mpmath.fsum(e)
+        for d in range(4):
+            want = mpmath.fsum(e[j] * mpmath.mpf(vd[j, d]) for j in range(4)) / z
+            assert abs(float(want) - o[0, 0, i, d]) <= 1e-14, (i, d)
+        assert abs(float(mpmath.log(z)) - lse[0, 0, i]) <= 1e-14
+
+
+def pin_large_logits_stable(orc):
+    """Logits of magnitude ~1000 neither overflow nor underflow (softmax shift invariance)."""
+    # q = 32 e_0 and k_j = c_j e_0: exact bf16 inputs with logits spread over 800
+    D = 8
+    q = np.zeros((1, 1, 1, D), dtype=np.float32)
+    q[..., 0] = 32.0
+    v = np.zeros((1, 1, 3, D), dtype=np.float32)
+    v[0, 0, :, 1] = [1.0, 2.0, 4.0]
+    for c in ([-18.75, 0.0, 6.25], [-30.0, -31.0, -31.5]):
+        k = np.zeros((1, 1, 3, D), dtype=np.float32)
+        k[0, 0, :, 0] = c
+        o, lse = orc.attn_fwd(_bits_of(q), _bits_of(k), _bits_of(v), 1.0)
+        s = 32.0 * np.array(c)
+        w = np.exp(s - s.max())
+        want_lse = s.max() + np.log(w.sum())
+        w /= w.sum()
+        assert np.all(np.isfinite(o)) and np.isfinite(lse).all()
+        np.testing.assert_allclose(o[0, 0, 0, 1], (w * [1, 2, 4]).sum(), rtol=0, atol=1e-13)
+        np.testing.assert_allclose(lse[0, 0, 0], want_lse, rtol=1e-15, atol=0)
+
+
+ALL_PINS = [pin_single_key, pin_two_keys, pin_weights_sum_to_one, pin_constant_values,
+            pin_zero_logits, pin_query_permutation, pin_key_value_permutation,
+            pin_value_translation, pin_varlen_is_truncation, pin_varlen_empty_and_clamped,
+            pin_row_subset, pin_torch_sdpa, pin_mpmath_brute_force, pin_large_logits_stable]

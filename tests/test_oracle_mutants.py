@@ -1,0 +1,93 @@
+"""Every plausible mistake planted in a copy of the oracle is caught by some pin.
+
+Each mutant is a textual edit of ``oracle/oracle.c`` (a dropped term, a wrong
+sign, index or operand), compiled to a temporary library and checked against
+the pins of ``oracle_pins.py`` in a child process (a mutant that reads out of
+bounds may crash; a crash counts as caught).  The real oracle is never edited.
+"""
+import os
+import subprocess
+import sys
+import tempfile
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+SOURCE = os.path.join(ROOT, "oracle", "oracle.c")
+
+MUTANTS = {
+    "scale_dropped": [("s[j] = scale * dot;", "s[j] = dot;")],
+    "scale_twice": [("s[j] = scale * dot;", "s[j] = scale * scale * dot;")],
+    "k_transposed": [("bf16_to_f64(k[(size_t)j * D + d])", "bf16_to_f64(k[(size_t)d * L + j])")],
+    "dot_skips_first_dim": [("for (int d = 0; d < D; ++d)\n            dot",
+                             "for (int d = 1; d < D; ++d)\n            dot")],
+    "lse_drops_max": [("*lse = m + log(l);", "*lse = log(l);")],
+    "lse_log2": [("*lse = m + log(l);", "*lse = m + log2(l);")],
+    "exp_sign": [("exp(s[j] - m)", "exp(m - s[j])")],
+    "no_max_shift": [("exp(s[j] - m)", "exp(s[j])"), ("*lse = m + log(l);", "*lse = log(l);")],
+    "min_not_max": [("if (s[j] > m)", "if (s[j] < m)")],
+    "not_normalised": [("double p = exp(s[j] - m) / l;", "double p = exp(s[j] - m);")],
+    "v_dims_reversed": [("bf16_to_f64(v[(size_t)j * D + d])", "bf16_to_f64(v[(size_t)j * D + (D - 1 - d)])")],
+    "varlen_off_by_one": [("int L = kv_lens[b];", "int L = kv_lens[b] + 1;")],
+    "varlen_wrong_sample": [("valid_len(kv_lens, b, Skv)", "valid_len(kv_lens, 0, Skv)")],
+    "rows_ignore_head": [("rows[bh * nrows + r]", "rows[r]")],
+    "q_ignores_head": [("((size_t)bh * Sq + i) * D", "((size_t)i) * D")],
+    "k_ignores_head": [("k + (size_t)bh * Skv * D", "k")],
+    "v_ignores_head": [("v + (size_t)bh * Skv * D", "v")],
+}
+
+CHILD = r"""
+import sys, traceback
+sys.path.insert(0, sys.argv[2]); sys.path.insert(0, sys.argv[3])
+import oracle, oracle_pins
+orc = oracle.Oracle(sys.argv[1])
+failed = []
+for pin in oracle_pins.ALL_PINS:
+    try:
+        pin(orc)
+    except Exception:
+        failed.append(pin.__name__)
+print("FAILED:" + ",".join(failed))
+"""
+
+
+def _mutate(text, edits):
+    for old, new in edits:
+        assert old in text, f"mutation anchor not found: {old!r}"
+        text = text.replace(old, new)
+    return text
+
+
+def test_real_oracle_passes_in_child(tmp_path):
+    import oracle
+    lib = oracle.build(output=str(tmp_path / "liboracle_real.so"))
+    out = subprocess.run([sys.executable, "-c", CHILD, lib, ROOT, os.path.join(ROOT, "tests")],
+                         capture_output=True, text=True, timeout=300)
+    assert out.returncode == 0, out.stderr
+    assert "FAILED:\n" in out.stdout or out.stdout.strip() == "FAILED:", out.stdout
+
+
+def test_every_mutant_is_caught():
+    import oracle
+    text = open(SOURCE).read()
+    procs = {}
+    with tempfile.TemporaryDirectory() as tmp:
+        for name, edits in MUTANTS.items():
+            src = os.path.join(tmp, f"{name}.c")
+            with open(src, "w") as f:
+                f.write(_mutate(text, edits))
+            lib = oracle.build(source=src, output=os.path.join(tmp, f"lib{name}.so"))
+            procs[name] = subprocess.Popen(
+                [sys.executable, "-c", CHILD, lib, ROOT, os.path.join(ROOT, "tests")],
+                stdout=subprocess.PIPE, stderr=subprocess.PIPE, text=True,
+                env={**os.environ, "OMP_NUM_THREADS": "1"})
+        survivors = []
+        for name, p in procs.items():
+            out, err = p.communicate(timeout=600)
+            caught = p.returncode != 0
+            if not caught:
+                line = [ln for ln in out.splitlines() if ln.startswith("FAILED:")]
+                caught = bool(line) and line[-1] != "FAILED:"
+            if not caught:
+                survivors.append(name)
+    assert not survivors, f"mutants not caught by any pin: {survivors}"
