@@ -1,0 +1,103 @@
+/*
+ * vdx.h -- C ABI of the GB300 (sm_103a) softmax attention forward library.
+ *
+ * The operation is the attention step of video diffusion-transformer
+ * inference described in the vidax paper (arXiv 2609.18077):
+ *   - Sec. 2, "3D RoPE, 3D VAEs, and flash attention": unmasked multi-head
+ *     attention over patchified spatiotemporal tokens, computed with a
+ *     flash-attention kernel so the Sq x Skv score matrix is never stored;
+ *   - Sec. 1: patchified video volumes give tens of thousands of tokens per
+ *     sample, so attention cost is quadratic in the token count;
+ *   - appendix Table 4 (porting-bug taxonomy): padded text tokens must be
+ *     excluded, by skipping invalid key blocks rather than by a dense
+ *     (B, H, Sq, Sk) mask -- the varlen entry point below.
+ *
+ * For each batch b, head h and query row i, with L valid keys:
+ *     s_j  = scale * <q[b,h,i,:], k[b,h,j,:]>,            j < L
+ *     out[b,h,i,:] = sum_j softmax(s)_j * v[b,h,j,:]
+ *     lse[b,h,i]   = ln(sum_j exp(s_j))                  (natural log)
+ * L = 0 gives out = 0 and lse = -inf.
+ *
+ * Conventions shared by every entry point:
+ *   - Tensors are contiguous, row-major, bf16 (IEEE bfloat16 bits):
+ *       q, out: [B, H, Sq, D];  k, v: [B, H, Skv, D];  lse: fp32 [B, H, Sq].
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the
+ *     library never frees or keeps them after the call returns, and it
+ *     allocates no device memory per call.
+ *   - q, k, v and out must be 16-byte aligned (TMA and vector stores); lse
+ *     4-byte aligned.  out must not overlap q, k or v.
+ *   - D must be 64 or 128.  B, H, Sq, Skv >= 0; B*H*Sq == 0 is a no-op.
+ *   - The call is asynchronous on `stream` (a cudaStream_t, NULL = the legacy
+ *     default stream) of the CURRENT device, which must be an sm_103 GPU.
+ *   - Arguments are validated before any CUDA work; a failing call returns a
+ *     vdx_status and launches nothing.  Nothing is thrown across the ABI and
+ *     the library never exits the process.
+ *   - Thread-safe: one-time per-device set-up is guarded internally.
+ */
+#ifndef VDX_H
+#define VDX_H
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum vdx_status {
+    VDX_OK = 0,
+    VDX_ERR_INVALID_ARG = 1, /* null pointer, negative size, bad D, size overflow */
+    VDX_ERR_UNSUPPORTED = 2, /* a shape outside what the kernel implements */
+    VDX_ERR_MISALIGNED = 3,  /* a pointer breaks the alignment rules above */
+    VDX_ERR_CUDA = 4,        /* a CUDA runtime/driver call failed */
+    VDX_ERR_DEVICE = 5,      /* the current device is not an sm_103 GPU */
+    VDX_ERR_TIMEOUT = 6      /* a bounded in-kernel wait expired (see vdx_check_device_error) */
+} vdx_status;
+
+/*
+ * Dense (non-causal, unmasked) attention forward, Sec. 2 of the paper.
+ *   q   : bf16 [B,H,Sq,D]          k, v : bf16 [B,H,Skv,D]
+ *   out : bf16 [B,H,Sq,D] written   lse  : fp32 [B,H,Sq] written, or NULL to skip
+ *   scale: logit multiplier (1/sqrt(D) for standard attention); any finite value.
+ * Skv == 0 writes out = 0 and lse = -inf.
+ */
+int vdx_attn_fwd(const void *q, const void *k, const void *v, void *out, float *lse,
+                 int B, int H, int Sq, int Skv, int D, float scale, void *stream);
+
+/*
+ * Cross-attention to padded text tokens (appendix Table 4: per-sample valid
+ * key counts instead of a dense mask).  As vdx_attn_fwd with Skv = Skv_max,
+ * except that sample b attends only to keys j < clamp(kv_lens[b], 0, Skv_max).
+ *   kv_lens: DEVICE int32 [B], caller-owned.  Key/value rows past a sample's
+ *            length are never used and may hold any bits, NaN included.
+ * Key tiles entirely past a sample's length are skipped, not masked.
+ */
+int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, float *lse,
+                        int B, int H, int Sq, int Skv_max, int D, const int *kv_lens,
+                        float scale, void *stream);
+
+/* Human-readable name of a vdx_status (static storage; never NULL). */
+const char *vdx_status_string(int status);
+
+/*
+ * Synchronises `stream`, then reads and clears the library's device error
+ * word on the current device.  Returns VDX_OK, VDX_ERR_TIMEOUT if a kernel
+ * gave up on a bounded wait since the last check, or VDX_ERR_CUDA if the
+ * synchronisation itself failed.
+ */
+int vdx_check_device_error(void *stream);
+
+/*
+ * Failure-detection self-test: launches one block whose only wait is on an
+ * mbarrier that nothing ever arrives on, bounded by `limit_us` microseconds
+ * (1 .. 10,000,000).  The kernel records VDX_ERR_TIMEOUT in the device error
+ * word and returns; the GPU context stays usable.  Read the result with
+ * vdx_check_device_error.  No fault, trap or hang is involved.
+ */
+int vdx_selftest_wait_timeout(int limit_us, void *stream);
+
+/* Library version as major*10000 + minor*100 + patch. */
+int vdx_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VDX_H */

@@ -1,1 +1,8 @@
-"""GB300-native (sm_103a) softmax attention forward for video-DiT inference."""
+"""GB300-native (sm_103a) softmax attention forward for video-DiT inference.
+
+The compute path is the CUDA library ``_lib/libvdx.so`` (C ABI in
+``include/vdx.h``); ``binding`` forwards torch tensors' device pointers to
+it.  The library is loaded on first use and its absence is an error.
+"""
+from .binding import (VdxError, attn_fwd, attn_fwd_varlen, check_device_error, load,  # noqa: F401
+                      selftest_wait_timeout, status_string, version)

@@ -1,0 +1,157 @@
+"""ctypes binding of libvdx (include/vdx.h): argument marshalling only.
+
+Every step of the attention forward runs in the CUDA library; this module
+checks tensor metadata, allocates outputs through PyTorch when the caller
+does not pass them, and forwards raw device pointers, sizes and the current
+CUDA stream.  There is no fallback: if the library is missing or the call
+fails, an exception is raised.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libvdx.so")
+
+VDX_OK = 0
+VDX_ERR_INVALID_ARG = 1
+VDX_ERR_UNSUPPORTED = 2
+VDX_ERR_MISALIGNED = 3
+VDX_ERR_CUDA = 4
+VDX_ERR_DEVICE = 5
+VDX_ERR_TIMEOUT = 6
+
+# Every symbol include/vdx.h declares, with its ctypes signature.
+_P = ctypes.c_void_p
+_I = ctypes.c_int
+SIGNATURES = {
+    "vdx_attn_fwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, ctypes.c_float, _P]),
+    "vdx_attn_fwd_varlen": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, ctypes.c_float, _P]),
+    "vdx_status_string": (ctypes.c_char_p, [_I]),
+    "vdx_check_device_error": (_I, [_P]),
+    "vdx_selftest_wait_timeout": (_I, [_I, _P]),
+    "vdx_version": (_I, []),
+}
+
+_lib = None
+
+
+class VdxError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__(f"{where}: {status_string(status)} (status {status})")
+
+
+def load() -> ctypes.CDLL:
+    """Load libvdx.so (built in-tree by ``__graft_entry__.build()``)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                f"CUDA library {LIB_PATH} is not built; run `python -c \"import __graft_entry__ as g; g.build()\"`")
+        lib = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+    return _lib
+
+
+def status_string(status: int) -> str:
+    return load().vdx_status_string(int(status)).decode()
+
+
+def version() -> int:
+    return int(load().vdx_version())
+
+
+def _stream_handle(device: torch.device):
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def check_device_error(device=None) -> int:
+    """Synchronise the current stream and read/clear the device error word."""
+    device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    with torch.cuda.device(device):
+        return int(load().vdx_check_device_error(_stream_handle(device)))
+
+
+def selftest_wait_timeout(limit_us: int, device=None) -> int:
+    """Launch the bounded-wait self-test kernel; returns the launch status."""
+    device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    with torch.cuda.device(device):
+        return int(load().vdx_selftest_wait_timeout(int(limit_us), _stream_handle(device)))
+
+
+def _check_qkv(q, k, v):
+    for name, t in (("q", q), ("k", k), ("v", v)):
+        if not isinstance(t, torch.Tensor) or not t.is_cuda:
+            raise TypeError(f"{name} must be a CUDA tensor")
+        if t.dtype != torch.bfloat16 or t.dim() != 4 or not t.is_contiguous():
+            raise TypeError(f"{name} must be a contiguous bf16 [B,H,S,D] tensor")
+    if k.shape != v.shape or q.shape[:2] != k.shape[:2] or q.shape[3] != k.shape[3]:
+        raise ValueError(f"shape mismatch q{tuple(q.shape)} k{tuple(k.shape)} v{tuple(v.shape)}")
+    if not (q.device == k.device == v.device):
+        raise ValueError("q, k, v must be on one device")
+
+
+def _outputs(q, out, lse, return_lse):
+    B, H, Sq, D = q.shape
+    if out is None:
+        out = torch.empty_like(q)
+    elif out.shape != q.shape or out.dtype != torch.bfloat16 or not out.is_contiguous() or out.device != q.device:
+        raise ValueError("out must be a contiguous bf16 tensor shaped like q on q's device")
+    if lse is None and return_lse:
+        lse = torch.empty((B, H, Sq), dtype=torch.float32, device=q.device)
+    elif lse is not None and (lse.shape != (B, H, Sq) or lse.dtype != torch.float32 or not lse.is_contiguous()
+                              or lse.device != q.device):
+        raise ValueError("lse must be a contiguous fp32 [B,H,Sq] tensor on q's device")
+    return out, lse
+
+
+def attn_fwd(q, k, v, scale=None, out=None, lse=None, return_lse=True):
+    """Softmax attention forward through ``vdx_attn_fwd``.
+
+    q: bf16 [B,H,Sq,D]; k, v: bf16 [B,H,Skv,D] (CUDA, contiguous).
+    scale defaults to 1/sqrt(D).  Returns (out bf16 [B,H,Sq,D], lse fp32 [B,H,Sq] or None).
+    """
+    _check_qkv(q, k, v)
+    B, H, Sq, D = q.shape
+    Skv = k.shape[2]
+    scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
+    out, lse = _outputs(q, out, lse, return_lse)
+    with torch.cuda.device(q.device):
+        st = load().vdx_attn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                                 lse.data_ptr() if lse is not None else None,
+                                 B, H, Sq, Skv, D, scale, _stream_handle(q.device))
+    if st != VDX_OK:
+        raise VdxError(st, "vdx_attn_fwd")
+    return out, lse
+
+
+def attn_fwd_varlen(q, k, v, kv_lens, scale=None, out=None, lse=None, return_lse=True):
+    """Cross-attention to padded keys through ``vdx_attn_fwd_varlen``.
+
+    kv_lens: int32 CUDA tensor [B] of valid key counts (keys past it are ignored).
+    """
+    _check_qkv(q, k, v)
+    B, H, Sq, D = q.shape
+    Skv_max = k.shape[2]
+    if (not isinstance(kv_lens, torch.Tensor) or kv_lens.dtype != torch.int32 or kv_lens.shape != (B,)
+            or kv_lens.device != q.device or not kv_lens.is_contiguous()):
+        raise TypeError("kv_lens must be a contiguous int32 CUDA tensor of shape [B] on q's device")
+    scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
+    out, lse = _outputs(q, out, lse, return_lse)
+    with torch.cuda.device(q.device):
+        st = load().vdx_attn_fwd_varlen(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                                        lse.data_ptr() if lse is not None else None,
+                                        B, H, Sq, Skv_max, D, kv_lens.data_ptr(), scale,
+                                        _stream_handle(q.device))
+    if st != VDX_OK:
+        raise VdxError(st, "vdx_attn_fwd_varlen")
+    return out, lse

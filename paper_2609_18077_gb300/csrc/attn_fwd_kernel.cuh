@@ -1,0 +1,507 @@
+// Softmax attention forward for sm_103a (GB300): TMA-fed, tcgen05 tensor cores,
+// accumulators and probabilities in tensor memory, warp-specialised.
+//
+// What it computes (vidax paper, Sec. 2 "3D RoPE, 3D VAEs, and flash
+// attention"): out = softmax(scale * Q K^T) V and the natural-log row
+// log-sum-exp, without ever storing the Sq x Skv score matrix, over
+// [B, H, S, D] bf16 video tokens.  The varlen instance skips key tiles past a
+// sample's valid text length and masks the ragged last tile (appendix Table 4:
+// segment-id masking of padded text keys instead of a dense mask).
+//
+// Work unit: one CTA owns one (b*h, pair of 128-row query tiles).  Roles:
+//   warps 0-3  softmax group 0: query tile 0, TMEM lane = query row
+//   warps 4-7  softmax group 1: query tile 1
+//   warp  8    TMA producer: Q tiles once, then K_0 V_0 K_1 V_1 ... through a
+//              ring of NSLOT shared-memory slots
+//   warp  9    tcgen05 issuer (one lane) and TMEM owner
+// Tensor memory (512 columns x 128 lanes, fp32):
+//   S_t = cols [128t, 128t+128): logits Q_t K_j^T; the probabilities P_t are
+//         written back over its first 64 columns as packed bf16 pairs and fed
+//         to the second GEMM straight from TMEM.
+//   O_t = cols [256+128t, 256+128t+D): the running output accumulator.
+// MMA order per key tile j (ping-pong between the two query tiles so that one
+// group's softmax overlaps the other group's GEMMs):
+//   ... PV_0(j)  S_0(j+1)  PV_1(j)  S_1(j+1) ...
+// Online softmax in base 2 with a lazy maximum: a row's reference maximum m
+// only moves when the tile maximum exceeds it by more than TAU (log2 units),
+// so p <= 2^TAU and the O rescale in TMEM is rare after the first tiles.
+//
+// Every wait is bounded (globaltimer); on expiry the CTA records
+// VDX_ERR_TIMEOUT in the device error word, skips the rest of its work, frees
+// its tensor memory and returns.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cstdint>
+
+#include "sm103_ptx.cuh"
+
+namespace vdx {
+
+// Device error word: bit 0 = a bounded wait expired.  Read and cleared by
+// vdx_check_device_error.
+__device__ unsigned int g_error_word;
+
+constexpr int BM = 128;          // query rows per tile (= TMEM lanes)
+constexpr int BN = 128;          // keys per tile
+constexpr int NUM_THREADS = 320; // 8 softmax warps + producer + MMA
+constexpr int PRODUCER_WARP = 8;
+constexpr int MMA_WARP = 9;
+constexpr float TAU = 8.0f;      // lazy-rescale threshold, log2 units
+constexpr uint32_t TMEM_COLS = 512;
+
+struct AttnParams {
+    __nv_bfloat16 *out;
+    float *lse;
+    const int *kv_lens;   // varlen only
+    int H;
+    int Sq;
+    int Skv;              // Skv (dense) or Skv_max (varlen)
+    int q_pairs;          // ceil(ceil(Sq / BM) / 2)
+    float scale_log2;     // scale * log2(e)
+    uint64_t wait_limit_ns;
+};
+
+template <int D>
+struct Layout {
+    static_assert(D == 64 || D == 128, "head dim");
+    static constexpr int TILE_BYTES = BM * D * 2;           // one Q, K or V tile
+    static constexpr int HALF_BYTES = BM * 128;              // one 64-column swizzle block
+    static constexpr int NSLOT = D == 128 ? 4 : 8;           // K/V ring
+    static constexpr int Q_OFF = 0;
+    static constexpr int KV_OFF = 2 * TILE_BYTES;
+    static constexpr int BAR_OFF = KV_OFF + NSLOT * TILE_BYTES;
+    // barrier indices
+    static constexpr int B_Q = 0;                            // [2] Q tile t landed
+    static constexpr int B_FULL = 2;                         // [NSLOT] slot landed
+    static constexpr int B_EMPTY = B_FULL + NSLOT;           // [NSLOT] slot consumed
+    static constexpr int B_S = B_EMPTY + NSLOT;              // [2] S_t ready
+    static constexpr int B_P = B_S + 2;                      // [2] P_t written, O_t rescaled
+    static constexpr int B_O = B_P + 2;                      // [2] last PV_t done
+    static constexpr int B_FIX = B_O + 2;                    // varlen V tile staging
+    static constexpr int B_DRAIN = B_FIX + 1;                // all MMAs retired
+    static constexpr int NBARS = B_DRAIN + 1;
+    static constexpr int TMEM_PTR_OFF = BAR_OFF + NBARS * 8;
+    static constexpr int ABORT_OFF = TMEM_PTR_OFF + 4;
+    static constexpr int BYTES = ABORT_OFF + 4;
+    static constexpr int ALLOC = BYTES + 1024;               // slack for 1024-B alignment
+};
+
+__device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                             uint64_t limit_ns)
+{
+    if (ptx::mbar_try_wait(bar, parity))
+        return true;
+    const uint64_t t0 = ptx::globaltimer_ns();
+    for (uint32_t n = 1;; ++n) {
+        if (ptx::mbar_try_wait(bar, parity))
+            return true;
+        if ((n & 255u) == 0) {
+            if (*abort_flag)
+                return false;
+            if (ptx::globaltimer_ns() - t0 > limit_ns) {
+                *abort_flag = 1;
+                atomicOr(&g_error_word, 1u);
+                return false;
+            }
+        }
+    }
+}
+
+__device__ __forceinline__ float ex2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
+{
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&v);
+}
+
+// S_t = Q_t K^T: M = 128 query rows, N = 128 keys, K = D in steps of 16.
+// Both operands K-major, 128-byte swizzle, stored as D/64 blocks of
+// 128 rows x 128 bytes; 8-row groups are 1024 bytes apart.
+template <int D>
+__device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint32_t q_smem, uint32_t k_smem)
+{
+    constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, BN, 0);
+#pragma unroll
+    for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = (kk >> 2) * Layout<D>::HALF_BYTES + (kk & 3) * 32;
+        ptx::mma_ss(s_tmem, ptx::smem_desc_sw128(q_smem + off, 16, 1024),
+                    ptx::smem_desc_sw128(k_smem + off, 16, 1024), idesc, kk > 0);
+    }
+}
+
+// O_t (+)= P_t V: M = 128, N = D, K = 128 keys in steps of 16.  P comes from
+// TMEM (16 bf16 = 8 columns per step); V is N-major ("MN-major"): each key row
+// holds 64 contiguous head-dim values per 128-byte swizzled row, the two
+// 64-column blocks are HALF_BYTES apart (LBO), 8-key groups 1024 bytes (SBO).
+template <int D>
+__device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint32_t v_smem, bool accumulate)
+{
+    constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, D, 1);
+#pragma unroll
+    for (int kk = 0; kk < BN / 16; ++kk) {
+        ptx::mma_ts(o_tmem, p_tmem + kk * 8, ptx::smem_desc_sw128(v_smem + kk * 2048, Layout<D>::HALF_BYTES, 1024),
+                    idesc, (accumulate || kk > 0) ? 1u : 0u);
+    }
+}
+
+// Row maximum (or minimum for a negative scale) of the raw logits, over the
+// first `valid` columns when PARTIAL.
+template <bool PARTIAL>
+__device__ __forceinline__ float tile_extreme(const uint32_t (&s)[4][32], bool neg_scale, int valid)
+{
+    float e0 = neg_scale ? INFINITY : -INFINITY, e1 = e0, e2 = e0, e3 = e0;
+#pragma unroll
+    for (int c = 0; c < BN; c += 4) {
+        float x0 = __uint_as_float(s[c >> 5][c & 31]);
+        float x1 = __uint_as_float(s[c >> 5][(c & 31) + 1]);
+        float x2 = __uint_as_float(s[c >> 5][(c & 31) + 2]);
+        float x3 = __uint_as_float(s[c >> 5][(c & 31) + 3]);
+        if (PARTIAL) {
+            const float pad = neg_scale ? INFINITY : -INFINITY;
+            x0 = c + 0 < valid ? x0 : pad;
+            x1 = c + 1 < valid ? x1 : pad;
+            x2 = c + 2 < valid ? x2 : pad;
+            x3 = c + 3 < valid ? x3 : pad;
+        }
+        if (neg_scale) {
+            e0 = fminf(e0, x0); e1 = fminf(e1, x1); e2 = fminf(e2, x2); e3 = fminf(e3, x3);
+        } else {
+            e0 = fmaxf(e0, x0); e1 = fmaxf(e1, x1); e2 = fmaxf(e2, x2); e3 = fmaxf(e3, x3);
+        }
+    }
+    return neg_scale ? fminf(fminf(e0, e1), fminf(e2, e3)) : fmaxf(fmaxf(e0, e1), fmaxf(e2, e3));
+}
+
+// p = 2^(x * scale_log2 - m) for the 128 logits of this row, packed to bf16
+// pairs (even column in the low half); returns the fp32 sum of the p values.
+template <bool PARTIAL>
+__device__ __forceinline__ float tile_probs(const uint32_t (&s)[4][32], uint32_t (&pk)[2][32], float sl2,
+                                            float neg_m, int valid)
+{
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+    for (int c = 0; c < BN; c += 4) {
+        float p0 = ex2(fmaf(__uint_as_float(s[c >> 5][(c & 31) + 0]), sl2, neg_m));
+        float p1 = ex2(fmaf(__uint_as_float(s[c >> 5][(c & 31) + 1]), sl2, neg_m));
+        float p2 = ex2(fmaf(__uint_as_float(s[c >> 5][(c & 31) + 2]), sl2, neg_m));
+        float p3 = ex2(fmaf(__uint_as_float(s[c >> 5][(c & 31) + 3]), sl2, neg_m));
+        if (PARTIAL) {
+            p0 = c + 0 < valid ? p0 : 0.f;
+            p1 = c + 1 < valid ? p1 : 0.f;
+            p2 = c + 2 < valid ? p2 : 0.f;
+            p3 = c + 3 < valid ? p3 : 0.f;
+        }
+        a0 += p0;
+        a1 += p1;
+        a2 += p2;
+        a3 += p3;
+        pk[c >> 6][(c & 63) >> 1] = pack_bf16x2(p0, p1);
+        pk[c >> 6][((c & 63) >> 1) + 1] = pack_bf16x2(p2, p3);
+    }
+    return (a0 + a1) + (a2 + a3);
+}
+
+template <int D, bool VARLEN>
+__global__ void __launch_bounds__(NUM_THREADS, 1)
+    attn_fwd_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
+                    const __grid_constant__ CUtensorMap tmap_v, const AttnParams p)
+{
+    using L = Layout<D>;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    const uint32_t sbase = ptx::smem_u32(sm);
+    auto bar = [&](int i) -> uint32_t { return sbase + L::BAR_OFF + 8 * i; };
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + L::ABORT_OFF);
+    const uint64_t limit = p.wait_limit_ns;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int bh = blockIdx.x / p.q_pairs;
+    const int qp = blockIdx.x - bh * p.q_pairs;
+    int kv_valid = p.Skv;
+    if (VARLEN) {
+        const int len = __ldg(p.kv_lens + bh / p.H);
+        kv_valid = len < 0 ? 0 : (len > p.Skv ? p.Skv : len);
+    }
+    const int n_kv = (kv_valid + BN - 1) / BN;
+
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(bar(L::B_Q + 0), 1);
+        ptx::mbar_init(bar(L::B_Q + 1), 1);
+        for (int i = 0; i < L::NSLOT; ++i) {
+            ptx::mbar_init(bar(L::B_FULL + i), 1);
+            ptx::mbar_init(bar(L::B_EMPTY + i), 1);
+        }
+        for (int t = 0; t < 2; ++t) {
+            ptx::mbar_init(bar(L::B_S + t), 1);
+            ptx::mbar_init(bar(L::B_P + t), 4 * 32);
+            ptx::mbar_init(bar(L::B_O + t), 1);
+        }
+        ptx::mbar_init(bar(L::B_FIX), 1);
+        ptx::mbar_init(bar(L::B_DRAIN), 1);
+        *abort_flag = 0;
+        ptx::fence_barrier_init();
+        ptx::fence_proxy_async_smem();
+    }
+    if (warp == MMA_WARP) {
+        ptx::tmem_alloc(sbase + L::TMEM_PTR_OFF, TMEM_COLS);
+        ptx::tmem_relinquish();
+    }
+    if (warp == PRODUCER_WARP && lane == 0) {
+        ptx::tma_prefetch_desc(&tmap_q);
+        ptx::tma_prefetch_desc(&tmap_k);
+        ptx::tma_prefetch_desc(&tmap_v);
+    }
+    ptx::tc_fence_before_sync();
+    __syncthreads();
+    ptx::tc_fence_after_sync();
+    const uint32_t tmem = *reinterpret_cast<volatile uint32_t *>(sm + L::TMEM_PTR_OFF);
+
+    if (warp == PRODUCER_WARP) {
+        // ------------------------------------------------------------ TMA producer
+        if (n_kv > 0) {
+            if (lane == 0) {
+                for (int t = 0; t < 2; ++t) {
+                    ptx::mbar_arrive_expect_tx(bar(L::B_Q + t), L::TILE_BYTES);
+                    for (int h = 0; h < D / 64; ++h)
+                        ptx::tma_load_3d(sbase + L::Q_OFF + t * L::TILE_BYTES + h * L::HALF_BYTES, &tmap_q,
+                                         bar(L::B_Q + t), h * 64, (qp * 2 + t) * BM, bh);
+                }
+            }
+            for (int it = 0; it < 2 * n_kv; ++it) {
+                const int slot = it % L::NSLOT;
+                if (it >= L::NSLOT) {
+                    if (!__all_sync(0xffffffffu,
+                                    wait_bounded(bar(L::B_EMPTY + slot), ((it / L::NSLOT) - 1) & 1, abort_flag, limit)))
+                        break;
+                }
+                const int j = it >> 1;
+                const bool is_v = it & 1;
+                const uint32_t dst = sbase + L::KV_OFF + slot * L::TILE_BYTES;
+                const CUtensorMap *tm = is_v ? &tmap_v : &tmap_k;
+                const int valid_in_tile = kv_valid - j * BN;
+                if (!(VARLEN && is_v && valid_in_tile < BN)) {
+                    if (lane == 0) {
+                        ptx::mbar_arrive_expect_tx(bar(L::B_FULL + slot), L::TILE_BYTES);
+                        for (int h = 0; h < D / 64; ++h)
+                            ptx::tma_load_3d(dst + h * L::HALF_BYTES, tm, bar(L::B_FULL + slot), h * 64, j * BN, bh);
+                    }
+                } else {
+                    // Last V tile of a padded sample: rows past the valid length
+                    // may hold any bits (NaN included) and 0 * NaN = NaN inside
+                    // the GEMM, so stage the tile, zero those rows, then publish.
+                    if (lane == 0) {
+                        ptx::mbar_arrive_expect_tx(bar(L::B_FIX), L::TILE_BYTES);
+                        for (int h = 0; h < D / 64; ++h)
+                            ptx::tma_load_3d(dst + h * L::HALF_BYTES, tm, bar(L::B_FIX), h * 64, j * BN, bh);
+                    }
+                    if (!__all_sync(0xffffffffu, wait_bounded(bar(L::B_FIX), 0, abort_flag, limit)))
+                        break;
+                    const int nrow = BN - valid_in_tile;
+                    const int per_half = nrow * 8;   // 16-byte chunks per 64-column block
+                    uint8_t *slot_ptr = sm + L::KV_OFF + slot * L::TILE_BYTES;
+                    for (int e = lane; e < per_half * (D / 64); e += 32) {
+                        const int h = e / per_half;
+                        const int rem = e - h * per_half;
+                        const int r = valid_in_tile + (rem >> 3);
+                        *reinterpret_cast<uint4 *>(slot_ptr + h * L::HALF_BYTES + r * 128 + (rem & 7) * 16) =
+                            make_uint4(0u, 0u, 0u, 0u);
+                    }
+                    ptx::fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0)
+                        ptx::mbar_arrive(bar(L::B_FULL + slot));
+                }
+            }
+        }
+    } else if (warp == MMA_WARP) {
+        // ------------------------------------------------------------ tcgen05 issuer
+        if (n_kv > 0 && lane == 0) {
+            const uint32_t q0 = sbase + L::Q_OFF;
+            const uint32_t q1 = q0 + L::TILE_BYTES;
+            const uint32_t s0 = tmem, s1 = tmem + 128, o0 = tmem + 256, o1 = tmem + 384;
+            auto slot_addr = [&](int it) { return sbase + L::KV_OFF + (it % L::NSLOT) * L::TILE_BYTES; };
+            auto full_wait = [&](int it) {
+                return wait_bounded(bar(L::B_FULL + it % L::NSLOT), (it / L::NSLOT) & 1, abort_flag, limit);
+            };
+            bool ok = wait_bounded(bar(L::B_Q + 0), 0, abort_flag, limit) &&
+                      wait_bounded(bar(L::B_Q + 1), 0, abort_flag, limit) && full_wait(0);
+            if (ok) {
+                ptx::tc_fence_after_sync();
+                issue_qk<D>(s0, q0, slot_addr(0));
+                ptx::mma_commit(bar(L::B_S + 0));
+                issue_qk<D>(s1, q1, slot_addr(0));
+                ptx::mma_commit(bar(L::B_S + 1));
+                ptx::mma_commit(bar(L::B_EMPTY + 0));
+                for (int j = 0; j < n_kv && ok; ++j) {
+                    const int itv = 2 * j + 1, itk = 2 * j + 2;
+                    const bool more = j + 1 < n_kv;
+                    ok = full_wait(itv) && wait_bounded(bar(L::B_P + 0), j & 1, abort_flag, limit);
+                    if (!ok)
+                        break;
+                    ptx::tc_fence_after_sync();
+                    issue_pv<D>(o0, s0, slot_addr(itv), j > 0);
+                    if (!more)
+                        ptx::mma_commit(bar(L::B_O + 0));
+                    if (more) {
+                        if (!(ok = full_wait(itk)))
+                            break;
+                        ptx::tc_fence_after_sync();
+                        issue_qk<D>(s0, q0, slot_addr(itk));
+                        ptx::mma_commit(bar(L::B_S + 0));
+                    }
+                    if (!(ok = wait_bounded(bar(L::B_P + 1), j & 1, abort_flag, limit)))
+                        break;
+                    ptx::tc_fence_after_sync();
+                    issue_pv<D>(o1, s1, slot_addr(itv), j > 0);
+                    ptx::mma_commit(bar(L::B_EMPTY + itv % L::NSLOT));
+                    if (!more)
+                        ptx::mma_commit(bar(L::B_O + 1));
+                    if (more) {
+                        issue_qk<D>(s1, q1, slot_addr(itk));
+                        ptx::mma_commit(bar(L::B_S + 1));
+                        ptx::mma_commit(bar(L::B_EMPTY + itk % L::NSLOT));
+                    }
+                }
+            }
+            // Retire every MMA this thread issued before TMEM is released.
+            ptx::mma_commit(bar(L::B_DRAIN));
+            const uint64_t t0 = ptx::globaltimer_ns();
+            while (!ptx::mbar_try_wait(bar(L::B_DRAIN), 0)) {
+                if (ptx::globaltimer_ns() - t0 > limit) {
+                    atomicOr(&g_error_word, 1u);
+                    break;
+                }
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ softmax groups
+        const int t = warp >> 2;                 // query tile of this group
+        const int wq = warp & 3;                 // TMEM lane quarter of this warp
+        const int q_row = (qp * 2 + t) * BM + wq * 32 + lane;
+        const uint32_t lane_addr = tmem + (static_cast<uint32_t>(wq * 32) << 16);
+        const uint32_t s_addr = lane_addr + 128 * t;
+        const uint32_t o_addr = lane_addr + 256 + 128 * t;
+        const float sl2 = p.scale_log2;
+        const bool neg_scale = sl2 < 0.f;
+        float m_used = -INFINITY;
+        float l = 0.f;
+        bool ok = true;
+
+        for (int j = 0; j < n_kv; ++j) {
+            if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_S + t), j & 1, abort_flag, limit))))
+                break;
+            ptx::tc_fence_after_sync();
+            uint32_t s[4][32];
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                ptx::tmem_ld32(s_addr + 32 * c, s[c]);
+            ptx::tmem_wait_ld();
+
+            const int valid = kv_valid - j * BN;
+            const bool partial = valid < BN;
+            const float ext = partial ? tile_extreme<true>(s, neg_scale, valid) : tile_extreme<false>(s, neg_scale, BN);
+            const float m_tile = ext * sl2;
+            const float m_new = fmaxf(m_used, m_tile);
+            const bool need = m_new > m_used + TAU;
+            float factor = 1.f;
+            if (need) {
+                factor = ex2(m_used - m_new);
+                m_used = m_new;
+            }
+            l *= factor;
+            uint32_t pk[2][32];
+            const float neg_m = -m_used;
+            l += partial ? tile_probs<true>(s, pk, sl2, neg_m, valid) : tile_probs<false>(s, pk, sl2, neg_m, BN);
+            ptx::tmem_st32(s_addr, pk[0]);
+            ptx::tmem_st32(s_addr + 32, pk[1]);
+            if (j > 0 && __any_sync(0xffffffffu, need)) {
+                // O_t is idle here: S_t(j) was committed after PV_t(j-1), and
+                // PV_t(j) waits for the arrive below.  Done after P so that the
+                // logits' registers are free.
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t r[32];
+                    ptx::tmem_ld32(o_addr + 32 * c, r);
+                    ptx::tmem_wait_ld();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i)
+                        r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
+                    ptx::tmem_st32(o_addr + 32 * c, r);
+                }
+            }
+            ptx::tmem_wait_st();
+            ptx::tc_fence_before_sync();
+            ptx::mbar_arrive(bar(L::B_P + t));
+        }
+
+        // ------------------------------------------------------------ epilogue
+        const bool store = q_row < p.Sq;
+        __nv_bfloat16 *orow = p.out + (static_cast<size_t>(bh) * p.Sq + (store ? q_row : 0)) * D;
+        if (n_kv == 0) {
+            if (store) {
+#pragma unroll
+                for (int c = 0; c < D / 8; ++c)
+                    reinterpret_cast<uint4 *>(orow)[c] = make_uint4(0u, 0u, 0u, 0u);
+                if (p.lse)
+                    p.lse[static_cast<size_t>(bh) * p.Sq + q_row] = -INFINITY;
+            }
+        } else if (ok && __all_sync(0xffffffffu, wait_bounded(bar(L::B_O + t), 0, abort_flag, limit))) {
+            ptx::tc_fence_after_sync();
+            const float inv_l = 1.f / l;
+#pragma unroll
+            for (int c = 0; c < D / 32; ++c) {
+                uint32_t r[32];
+                ptx::tmem_ld32(o_addr + 32 * c, r);
+                ptx::tmem_wait_ld();
+                uint32_t w[16];
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    w[i] = pack_bf16x2(__uint_as_float(r[2 * i]) * inv_l, __uint_as_float(r[2 * i + 1]) * inv_l);
+                if (store) {
+                    uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * c);
+#pragma unroll
+                    for (int v = 0; v < 4; ++v)
+                        dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+                }
+            }
+            if (store && p.lse)
+                p.lse[static_cast<size_t>(bh) * p.Sq + q_row] = (m_used + __log2f(l)) * 0.69314718055994530942f;
+        }
+    }
+
+    ptx::tc_fence_before_sync();
+    __syncthreads();
+    if (warp == MMA_WARP) {
+        ptx::tc_fence_after_sync();
+        ptx::tmem_dealloc(tmem, TMEM_COLS);
+    }
+}
+
+// Failure-detection self-test: one thread waits on a barrier nothing arrives on.
+__global__ void wait_timeout_selftest_kernel(uint64_t limit_ns)
+{
+    __shared__ __align__(8) uint64_t barrier_word;
+    __shared__ int abort_word;
+    const uint32_t b = ptx::smem_u32(&barrier_word);
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(b, 1);
+        abort_word = 0;
+        ptx::fence_barrier_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0)
+        (void)wait_bounded(b, 0, &abort_word, limit_ns);
+    __syncthreads();
+}
+
+}  // namespace vdx

@@ -1,0 +1,240 @@
+// Host side of libvdx: the C ABI declared in include/vdx.h.
+//
+// Validation happens before any CUDA call; then, once per device, the device
+// is checked to be sm_103 and the kernels' shared-memory limits are raised;
+// then three 3-D TMA tensor maps (head dim, sequence, batch*head) are encoded
+// and one kernel is launched on the caller's stream.  Nothing is allocated.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <climits>
+#include <cmath>
+#include <cstdint>
+#include <mutex>
+
+#include "attn_fwd_kernel.cuh"
+#include "vdx.h"
+
+namespace {
+
+constexpr int kVersion = 1 * 10000 + 0 * 100 + 0;
+constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per in-kernel wait
+constexpr int kMaxDevices = 64;
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    });
+    return fn;
+}
+
+struct DeviceState {
+    std::once_flag once;
+    int status = VDX_OK;
+};
+DeviceState g_devices[kMaxDevices];
+
+template <int D, bool VARLEN>
+cudaError_t raise_smem_limit()
+{
+    return cudaFuncSetAttribute(vdx::attn_fwd_kernel<D, VARLEN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                vdx::Layout<D>::ALLOC);
+}
+
+// One-time per-device check and kernel attribute set-up (current device).
+int device_ready()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices)
+        return VDX_ERR_UNSUPPORTED;
+    DeviceState &st = g_devices[dev];
+    std::call_once(st.once, [&] {
+        int major = 0, minor = 0;
+        if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+            cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess) {
+            st.status = VDX_ERR_CUDA;
+            return;
+        }
+        if (major != 10 || minor != 3) {
+            st.status = VDX_ERR_DEVICE;
+            return;
+        }
+        if (raise_smem_limit<64, false>() != cudaSuccess || raise_smem_limit<64, true>() != cudaSuccess ||
+            raise_smem_limit<128, false>() != cudaSuccess || raise_smem_limit<128, true>() != cudaSuccess) {
+            st.status = VDX_ERR_CUDA;
+            return;
+        }
+        st.status = encode_fn() ? VDX_OK : VDX_ERR_CUDA;
+    });
+    return st.status;
+}
+
+// [B*H, rows, D] bf16 tensor as a 3-D TMA map with 64 x 128 x 1 boxes, 128-B swizzle.
+int make_map(CUtensorMap *map, const void *base, long long rows, long long bh, int D)
+{
+    const cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(rows),
+                                static_cast<cuuint64_t>(bh)};
+    const cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(rows) * D * 2};
+    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(vdx::BM), 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    const CUresult r = encode_fn()(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides,
+                                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? VDX_OK : VDX_ERR_CUDA;
+}
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+bool overlaps(const void *a, size_t na, const void *b, size_t nb)
+{
+    const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+    return x < y + nb && y < x + na;
+}
+
+int attn_launch(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
+                int D, const int *kv_lens, bool varlen, float scale, void *stream)
+{
+    // ---- validation (no CUDA calls)
+    if (!q || !k || !v || !out || (varlen && !kv_lens))
+        return VDX_ERR_INVALID_ARG;
+    if (B < 0 || H < 0 || Sq < 0 || Skv < 0)
+        return VDX_ERR_INVALID_ARG;
+    if (D != 64 && D != 128)
+        return VDX_ERR_INVALID_ARG;
+    if (!std::isfinite(scale))
+        return VDX_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(out, 16) || (lse && !aligned(lse, 4)) ||
+        (kv_lens && !aligned(kv_lens, 4)))
+        return VDX_ERR_MISALIGNED;
+    const long long bh = static_cast<long long>(B) * H;
+    if (bh == 0 || Sq == 0)
+        return VDX_OK;
+    if (bh > INT_MAX)
+        return VDX_ERR_INVALID_ARG;
+    const long long q_tiles = (Sq + vdx::BM - 1) / vdx::BM;
+    const long long q_pairs = (q_tiles + 1) / 2;
+    if (bh * q_pairs > INT_MAX)
+        return VDX_ERR_UNSUPPORTED;
+    const size_t q_bytes = static_cast<size_t>(bh) * Sq * D * 2;
+    const size_t kv_bytes = static_cast<size_t>(bh) * Skv * D * 2;
+    if (overlaps(out, q_bytes, q, q_bytes) || (kv_bytes && (overlaps(out, q_bytes, k, kv_bytes) ||
+                                                           overlaps(out, q_bytes, v, kv_bytes))))
+        return VDX_ERR_INVALID_ARG;
+
+    // ---- device set-up
+    int st = device_ready();
+    if (st != VDX_OK)
+        return st;
+
+    CUtensorMap mq, mk, mv;
+    const long long kv_rows = Skv > 0 ? Skv : 1;   // never loaded when Skv == 0
+    if ((st = make_map(&mq, q, Sq, bh, D)) != VDX_OK || (st = make_map(&mk, k, kv_rows, bh, D)) != VDX_OK ||
+        (st = make_map(&mv, v, kv_rows, bh, D)) != VDX_OK)
+        return st;
+
+    vdx::AttnParams p{};
+    p.out = static_cast<__nv_bfloat16 *>(out);
+    p.lse = lse;
+    p.kv_lens = kv_lens;
+    p.H = H;
+    p.Sq = Sq;
+    p.Skv = Skv;
+    p.q_pairs = static_cast<int>(q_pairs);
+    p.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
+    p.wait_limit_ns = kWaitLimitNs;
+
+    const dim3 grid(static_cast<unsigned>(bh * q_pairs));
+    const dim3 block(vdx::NUM_THREADS);
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (D == 128) {
+        if (varlen)
+            vdx::attn_fwd_kernel<128, true><<<grid, block, vdx::Layout<128>::ALLOC, s>>>(mq, mk, mv, p);
+        else
+            vdx::attn_fwd_kernel<128, false><<<grid, block, vdx::Layout<128>::ALLOC, s>>>(mq, mk, mv, p);
+    } else {
+        if (varlen)
+            vdx::attn_fwd_kernel<64, true><<<grid, block, vdx::Layout<64>::ALLOC, s>>>(mq, mk, mv, p);
+        else
+            vdx::attn_fwd_kernel<64, false><<<grid, block, vdx::Layout<64>::ALLOC, s>>>(mq, mk, mv, p);
+    }
+    const cudaError_t e = cudaGetLastError();
+    if (e == cudaErrorNoKernelImageForDevice)
+        return VDX_ERR_DEVICE;
+    return e == cudaSuccess ? VDX_OK : VDX_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+int vdx_attn_fwd(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
+                 int D, float scale, void *stream)
+{
+    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, nullptr, false, scale, stream);
+}
+
+int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,
+                        int Skv_max, int D, const int *kv_lens, float scale, void *stream)
+{
+    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv_max, D, kv_lens, true, scale, stream);
+}
+
+const char *vdx_status_string(int status)
+{
+    switch (status) {
+    case VDX_OK: return "VDX_OK";
+    case VDX_ERR_INVALID_ARG: return "VDX_ERR_INVALID_ARG: invalid argument";
+    case VDX_ERR_UNSUPPORTED: return "VDX_ERR_UNSUPPORTED: shape not supported";
+    case VDX_ERR_MISALIGNED: return "VDX_ERR_MISALIGNED: pointer alignment";
+    case VDX_ERR_CUDA: return "VDX_ERR_CUDA: CUDA call failed";
+    case VDX_ERR_DEVICE: return "VDX_ERR_DEVICE: current device is not sm_103";
+    case VDX_ERR_TIMEOUT: return "VDX_ERR_TIMEOUT: bounded in-kernel wait expired";
+    default: return "unknown vdx status";
+    }
+}
+
+int vdx_check_device_error(void *stream)
+{
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    unsigned int word = 0;
+    if (cudaMemcpyFromSymbol(&word, vdx::g_error_word, sizeof word) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    if (word != 0) {
+        const unsigned int zero = 0;
+        if (cudaMemcpyToSymbol(vdx::g_error_word, &zero, sizeof zero) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        return VDX_ERR_TIMEOUT;
+    }
+    return VDX_OK;
+}
+
+int vdx_selftest_wait_timeout(int limit_us, void *stream)
+{
+    if (limit_us < 1 || limit_us > 10000000)
+        return VDX_ERR_INVALID_ARG;
+    const int st = device_ready();
+    if (st != VDX_OK)
+        return st;
+    vdx::wait_timeout_selftest_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(
+        static_cast<uint64_t>(limit_us) * 1000ull);
+    return cudaGetLastError() == cudaSuccess ? VDX_OK : VDX_ERR_CUDA;
+}
+
+int vdx_version(void) { return kVersion; }
+
+}  // extern "C"

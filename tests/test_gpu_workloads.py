@@ -1,0 +1,41 @@
+"""Parity on the five video-shaped workloads at full size, in the bench's launch
+configuration, against the oracle on a seeded subset of query rows per head.
+
+The subset is the first VDX_PARITY_ROWS (default 1024) of the workload's
+4096 seeded rows per (b, h); VDX_PARITY_ROWS=4096 checks all of them.
+"""
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from parity import compare, run_gpu, run_oracle
+
+pytestmark = pytest.mark.gpu
+
+ROWS = int(os.environ.get("VDX_PARITY_ROWS", "1024"))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_18077_gb300 import build, binding
+    build.build()
+    binding.load()
+
+
+@pytest.mark.parametrize("name", ["tiny", "small480", "cross", "large480", "large720"])
+def test_workload(name):
+    from paper_2609_18077_gb300 import workloads
+    w = workloads.generate(name)
+    rows = w["rows"]
+    if rows is not None:
+        rows = np.ascontiguousarray(rows[:, :ROWS])
+    out, lse = run_gpu(w["q"], w["k"], w["v"], w["scale"], w["kv_lens"])
+    o_ref, lse_ref = run_oracle(w["q"], w["k"], w["v"], w["scale"], w["kv_lens"], rows)
+    stats = compare(out, lse, o_ref, lse_ref, rows)
+    print(f"{name}: O max {stats[0]:.3e} mean {stats[1]:.3e} LSE rel {stats[2]:.3e}")
+    del out, lse
+    torch.cuda.empty_cache()

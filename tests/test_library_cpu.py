@@ -1,0 +1,83 @@
+"""The C-ABI library loads, exports every declared symbol, and validates
+arguments before any CUDA call (CPU only: no compute is launched)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "vdx.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_18077_gb300 import build, binding
+    build.build()
+    return binding.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(vdx_[a-z0-9_]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(lib):
+    from paper_2609_18077_gb300 import binding
+    names = declared_functions()
+    assert names, "no declarations found"
+    for n in names:
+        assert hasattr(lib, n), f"missing export {n}"
+    assert sorted(binding.SIGNATURES) == names
+
+
+def test_version_and_status(lib):
+    from paper_2609_18077_gb300 import binding
+    assert binding.version() == 10000
+    for s in range(7):
+        assert binding.status_string(s).startswith("VDX_")
+    assert binding.status_string(99) == "unknown vdx status"
+
+
+A = 0x10000  # fake, 16-byte aligned addresses: validation must reject before touching them
+GOOD = dict(q=A, k=2 * A, v=3 * A, out=4 * A, lse=5 * A, B=1, H=1, Sq=8, Skv=8, D=128, scale=0.1)
+
+
+def call(lib, **kw):
+    a = {**GOOD, **kw}
+    return lib.vdx_attn_fwd(a["q"], a["k"], a["v"], a["out"], a["lse"], a["B"], a["H"], a["Sq"], a["Skv"],
+                            a["D"], a["scale"], None)
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(q=None), 1), (dict(k=None), 1), (dict(v=None), 1), (dict(out=None), 1),
+    (dict(D=96), 1), (dict(D=0), 1), (dict(B=-1), 1), (dict(Sq=-2), 1), (dict(Skv=-1), 1),
+    (dict(scale=float("nan")), 1), (dict(scale=float("inf")), 1),
+    (dict(q=A + 8), 3), (dict(out=4 * A + 2), 3), (dict(lse=5 * A + 2), 3),
+    (dict(out=A), 1),                     # out overlaps q
+    (dict(B=0), 0), (dict(Sq=0), 0), (dict(H=0), 0),   # empty: no-op, no CUDA call
+])
+def test_validation(lib, kw, status):
+    assert call(lib, **kw) == status
+
+
+def test_varlen_requires_lengths(lib):
+    g = GOOD
+    assert lib.vdx_attn_fwd_varlen(g["q"], g["k"], g["v"], g["out"], g["lse"], 1, 1, 8, 8, 128, None,
+                                   0.1, None) == 1
+    assert lib.vdx_attn_fwd_varlen(g["q"], g["k"], g["v"], g["out"], g["lse"], 1, 1, 8, 8, 128, 6 * A + 1,
+                                   0.1, None) == 3
+
+
+def test_selftest_limit_validation(lib):
+    assert lib.vdx_selftest_wait_timeout(0, None) == 1
+    assert lib.vdx_selftest_wait_timeout(10000001, None) == 1
+
+
+def test_binding_rejects_cpu_tensors():
+    import torch
+    from paper_2609_18077_gb300 import binding
+    x = torch.zeros(1, 1, 4, 64, dtype=torch.bfloat16)
+    with pytest.raises(TypeError):
+        binding.attn_fwd(x, x, x)
