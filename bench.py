@@ -1,0 +1,375 @@
+"""Attention-forward benchmark on GB300: TFLOP/s, ms per call, roofline fraction.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+One step = one attention forward (one vdx_attn_fwd / vdx_attn_fwd_varlen
+launch) over the whole workload, inputs resident in HBM.  The default
+workload is the small-DiT 480p self-attention (B=1, H=12, D=128,
+S = 21*30*52 = 32760 tokens, logit std ~3).  FLOPs = 4*B*H*Sq*Skv*D
+(effective key counts for the padded-text workload).
+
+Timing: W untimed warm-up steps, then K steps bracketed by a barrier and a
+device synchronisation, timed with CUDA events on the launching stream; the
+max over ranks is reported.  Inputs (Q, K, V, O: 403 MB) exceed the 129 MB
+L2, so no flush is inserted.  SM clocks are sampled with nvidia-smi during
+the timed region.  A second timed pass ("e2e") goes through the same C ABI
+with pinned host buffers: every step copies Q, K, V host->device, runs the
+kernel and copies O and LSE back.
+
+--impl reference times the fp64 CPU oracle (the only reference this
+method has) on a bounded row sample of the same workload.  Under torchrun
+(N > 1) each rank runs its own copy of the workload (independent problems:
+weak scaling, no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import io
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "attention fwd TFLOP/s and ms/call at 1 GB300; fraction of dense bf16 peak"
+UNIT = "TFLOP/s"
+FALLBACK_PEAKS = {"bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "hbm_gbs": 6800.0}
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return d, "measured"
+    return dict(FALLBACK_PEAKS), "fallback"
+
+
+def dist_env():
+    return int(os.environ.get("RANK", "0")), int(os.environ.get("WORLD_SIZE", "1")), \
+        int(os.environ.get("LOCAL_RANK", "0"))
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason sampling around the timed region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int, log_path: str | None = None):
+        self.index = index
+        self.proc = None
+        self.log_path = log_path
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        self.text = ""
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.text, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.text, _ = self.proc.communicate()
+        if self.log_path:
+            with open(self.log_path, "w") as f:
+                f.write(self.text)
+        return False
+
+    def summary(self, max_mhz_hint=None):
+        rows = [r for r in csv.reader(io.StringIO(self.text)) if len(r) >= 9]
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            try:
+                sm.append(float(r[1]))
+                mx.append(float(r[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, r[5:9]):
+                if val.strip().lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": max_mhz_hint, "reasons": [], "samples": 0}
+        # samples under load: the timed region dominates the window
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx) if mx else max_mhz_hint,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def make_inputs(name):
+    from paper_2609_18077_gb300 import workloads
+    w = workloads.generate(name)
+    flops = w["workload"].flops(w["kv_lens"])
+    return w, flops
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2609_18077_gb300 import binding
+
+    rank, world, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=dev)
+
+    w, flops = make_inputs(args.workload)
+    wl = w["workload"]
+    q, k, v = (t.to(dev) for t in (w["q"], w["k"], w["v"]))
+    lens = None if w["kv_lens"] is None else torch.from_numpy(w["kv_lens"]).to(dev)
+    out = torch.empty_like(q)
+    lse = torch.empty(q.shape[:3], dtype=torch.float32, device=dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        if lens is None:
+            binding.attn_fwd(q, k, v, scale=wl.scale, out=out, lse=lse)
+        else:
+            binding.attn_fwd_varlen(q, k, v, lens, scale=wl.scale, out=out, lse=lse)
+
+    def barrier():
+        if world > 1:
+            dist.barrier(device_ids=[local])
+        torch.cuda.synchronize(dev)
+
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    for _ in range(args.warmup):
+        step()
+    st = binding.check_device_error(dev)
+    if st != binding.VDX_OK:
+        raise RuntimeError(binding.status_string(st))
+
+    # ---- device-resident timed region
+    peaks, peak_kind = load_peaks()
+    clocks_log = os.path.join(ROOT, "gpurun_out", "bench_clocks.csv") if os.path.isdir(
+        os.path.join(ROOT, "gpurun_out")) else None
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local, clocks_log) as clk:
+        barrier()
+        start.record(stream)
+        for _ in range(args.steps):
+            step()
+        end.record(stream)
+        barrier()
+    ms_total = max_over_ranks(start.elapsed_time(end))
+    st = binding.check_device_error(dev)
+    if st != binding.VDX_OK:
+        raise RuntimeError(binding.status_string(st))
+    ms_step = ms_total / args.steps
+    tflops = flops * world / (ms_step * 1e-3) / 1e12
+    per_launch_tflops = flops / (ms_step * 1e-3) / 1e12
+
+    # ---- end to end through the C ABI with pinned host buffers
+    qh, kh, vh = (t.pin_memory() for t in (w["q"], w["k"], w["v"]))
+    lh = None if w["kv_lens"] is None else torch.from_numpy(w["kv_lens"]).pin_memory()
+    oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    lseh = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
+    h2d = sum(t.numel() * t.element_size() for t in (qh, kh, vh)) + (0 if lh is None else lh.numel() * 4)
+    d2h = oh.numel() * oh.element_size() + lseh.numel() * lseh.element_size()
+
+    def e2e_step():
+        q.copy_(qh, non_blocking=True)
+        k.copy_(kh, non_blocking=True)
+        v.copy_(vh, non_blocking=True)
+        if lh is not None:
+            lens.copy_(lh, non_blocking=True)
+        step()
+        oh.copy_(out, non_blocking=True)
+        lseh.copy_(lse, non_blocking=True)
+
+    e2e_steps = max(3, min(args.steps, 50))
+    for _ in range(2):
+        e2e_step()
+    barrier()
+    s2, e2 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s2.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    e2.record(stream)
+    barrier()
+    e2e_ms = max_over_ranks(s2.elapsed_time(e2)) / e2e_steps
+    e2e_tflops = flops * world / (e2e_ms * 1e-3) / 1e12
+
+    # ---- oracle on the host cores (rank 0, N = 1 only)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = time_oracle(w, target_s=args.cpu_seconds)
+
+    if world > 1:
+        dist.destroy_process_group()
+    if rank != 0:
+        return
+
+    clocks = clk.summary(peaks.get("sm_max_mhz"))
+    peak = float(peaks["bf16_tflops"])
+    traffic = load_traffic(args.workload)
+    line = {
+        "metric": METRIC, "value": round(tflops, 2), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded N(0,1) bf16 tensors shaped like the workload; no dataset)",
+        "config": {"workload": wl.name, "description": wl.description, "B": wl.B, "H": wl.H,
+                   "Sq": wl.Sq, "Skv": wl.Skv, "D": wl.D, "scale": wl.scale,
+                   "flops_per_call": flops,
+                   "l2": "inputs larger than L2 (no flush): Q+K+V+O = %.0f MB" % (
+                       4 * q.numel() * 2 / 1e6 if lens is None else (2 * q.numel() + 2 * k.numel()) * 2 / 1e6),
+                   "parallelism": f"replicas x{world} (independent problems per GPU)"},
+        "clocks": clocks,
+        "e2e": {"value": round(e2e_tflops, 2), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "gpu_launches": args.steps,
+        "roofline": {"bound": "tensor", "achieved": round(per_launch_tflops, 2), "peak": peak,
+                     "unit": "TFLOP/s", "frac": round(per_launch_tflops / peak, 4),
+                     "peak_kind": f"{peak_kind} bf16 dense burst",
+                     "frac_of_sustained": round(per_launch_tflops / float(peaks["bf16_tflops_sustained"]), 4),
+                     "traffic": traffic,
+                     "kernel": "vdx::attn_fwd_kernel<%d,%s>" % (wl.D, "true" if lens is not None else "false")},
+        "cpu_baseline": cpu,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def load_traffic(workload):
+    """DRAM bytes per launch from a committed ncu summary, when one matches the current kernel."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f)
+    entry = d.get(workload)
+    if not entry:
+        return None
+    return entry.get("dram_bytes_per_launch")
+
+
+class OracleTimer:
+    """Times the fp64 oracle on seeded query-row samples of a workload.
+
+    calibrate() picks the rows per (b, h) that take about target_s seconds;
+    run() times one such sample and returns the cpu_baseline record.
+    """
+
+    def __init__(self, w, threads=0):
+        import oracle
+        from paper_2609_18077_gb300 import workloads
+        self.orc = oracle.default()
+        self.cores = self.orc.set_threads(threads)
+        self.w = w
+        wl = w["workload"]
+        self.wl = wl
+        self.bits = tuple(workloads.bf16_bits(w[n]) for n in ("q", "k", "v"))
+        self.rng = np.random.default_rng(wl.seed)
+        lens = w["kv_lens"]
+        keys = wl.Skv if lens is None else float(np.mean(np.clip(lens, 0, wl.Skv)))
+        self.flops_per_row = 4.0 * keys * wl.D
+        self.bh = wl.B * wl.H
+        self.n = 1
+
+    def _time(self, n):
+        rows = np.stack([np.sort(self.rng.choice(self.wl.Sq, size=n, replace=False))
+                         for _ in range(self.bh)]).astype(np.int32)
+        t0 = time.perf_counter()
+        self.orc.attn_fwd(*self.bits, self.wl.scale, kv_lens=self.w["kv_lens"], rows=rows)
+        return time.perf_counter() - t0
+
+    def calibrate(self, target_s):
+        n, dt = 1, self._time(1)
+        while dt < 0.25 and n < self.wl.Sq:
+            n = min(self.wl.Sq, n * 4)
+            dt = self._time(n)
+        self.n = int(min(self.wl.Sq, max(1, math.ceil(n * target_s / max(dt, 1e-6)))))
+        return self.n
+
+    def run(self):
+        dt = self._time(self.n)
+        flops = self.flops_per_row * self.n * self.bh
+        return {"value": round(flops / dt / 1e12, 6), "unit": UNIT, "cores": self.cores, "kind": "oracle",
+                "seconds": round(dt, 3),
+                "sample": f"{self.n} seeded query rows per (b,h) x {self.bh} (b,h) pairs of workload "
+                          f"{self.wl.name} ({flops:.3e} FLOP in fp64, OpenMP)"}
+
+
+def time_oracle(w, target_s=15.0):
+    t = OracleTimer(w)
+    t.calibrate(target_s)
+    return t.run()
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    w, flops = make_inputs(args.workload)
+    wl = w["workload"]
+    timer = OracleTimer(w)
+    per_step = min(5.0, max(0.2, args.cpu_seconds * 4 / max(1, args.steps + args.warmup)))
+    timer.calibrate(per_step)
+    for _ in range(args.warmup):
+        timer.run()
+    recs = [timer.run() for _ in range(args.steps)]
+    value = statistics.median(r["value"] for r in recs)
+    ms_per_step = flops / (value * 1e12) * 1e3
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded N(0,1) bf16 tensors shaped like the workload; no dataset)",
+        "config": {"workload": wl.name, "B": wl.B, "H": wl.H, "Sq": wl.Sq, "Skv": wl.Skv, "D": wl.D,
+                   "flops_per_call": flops,
+                   "note": "each step times the oracle on a bounded row sample; ms_per_step is the "
+                           "full call extrapolated from the sampled rate"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": recs[-1]["cores"], "kind": "oracle",
+                         "sample": recs[-1]["sample"] + " per step"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+        "gpu_launches": 0,
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    from paper_2609_18077_gb300 import workloads
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--workload", default=workloads.DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        print("note: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

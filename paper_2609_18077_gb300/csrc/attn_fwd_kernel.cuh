@@ -9,8 +9,8 @@
 // segment-id masking of padded text keys instead of a dense mask).
 //
 // Work unit: one CTA owns one (b*h, pair of 128-row query tiles).  Roles:
-//   warps 0-3  softmax group 0: query tile 0, TMEM lane = query row
-//   warps 4-7  softmax group 1: query tile 1
+//   warps 0-3  softmax of query tile 0: thread = one query row (TMEM lane)
+//   warps 4-7  softmax of query tile 1
 //   warp  8    TMA producer: Q tiles once, then K_0 V_0 K_1 V_1 ... through a
 //              ring of NSLOT shared-memory slots
 //   warp  9    tcgen05 issuer (one lane) and TMEM owner
@@ -19,12 +19,20 @@
 //         written back over its first 64 columns as packed bf16 pairs and fed
 //         to the second GEMM straight from TMEM.
 //   O_t = cols [256+128t, 256+128t+D): the running output accumulator.
-// MMA order per key tile j (ping-pong between the two query tiles so that one
-// group's softmax overlaps the other group's GEMMs):
+// MMA order per key tile j (ping-pong between the two query tiles so that the
+// softmax of one tile overlaps the GEMMs of the other):
 //   ... PV_0(j)  S_0(j+1)  PV_1(j)  S_1(j+1) ...
 // Online softmax in base 2 with a lazy maximum: a row's reference maximum m
 // only moves when the tile maximum exceeds it by more than TAU (log2 units),
 // so p <= 2^TAU and the O rescale in TMEM is rare after the first tiles.
+//
+// Normalisation.  The P V GEMM multiplies V by bf16-rounded weights r_j while
+// the softmax sums the fp32 weights p_j.  In a row dominated by one key the
+// mismatch r/p - 1 (up to 2^-8) would pass straight into O, so the divisor of
+// O is the exact sum plus, for every key tile, the rounding residual r - p of
+// that tile's largest weight in the row.  That makes the dominant weight
+// exact at the cost of a few instructions per tile; the log-sum-exp uses the
+// exact sum alone.
 //
 // Every wait is bounded (globaltimer); on expiry the CTA records
 // VDX_ERR_TIMEOUT in the device error word, skips the rest of its work, frees
@@ -122,87 +130,130 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
     return *reinterpret_cast<uint32_t *>(&v);
 }
 
+__device__ __forceinline__ float round_bf16(float x)
+{
+    return __bfloat162float(__float2bfloat16_rn(x));
+}
+
+__device__ __forceinline__ float max3(float a, float b, float c)
+{
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+__device__ __forceinline__ float min3(float a, float b, float c)
+{
+    float d;
+    asm("min.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
+// (d0, d1) = (a0, a1) * b + c on the paired fp32 datapath.
+__device__ __forceinline__ void ffma2(float &d0, float &d1, float a0, float a1, float b, float c)
+{
+    asm("{\n\t.reg .b64 ra, rb, rc;\n\t"
+        "mov.b64 ra, {%2, %3};\n\t"
+        "mov.b64 rb, {%4, %4};\n\t"
+        "mov.b64 rc, {%5, %5};\n\t"
+        "fma.rn.f32x2 ra, ra, rb, rc;\n\t"
+        "mov.b64 {%0, %1}, ra;\n\t}"
+        : "=f"(d0), "=f"(d1)
+        : "f"(a0), "f"(a1), "f"(b), "f"(c));
+}
+
+// (a0, a1) += (b0, b1) on the paired fp32 datapath.
+__device__ __forceinline__ void fadd2(float &a0, float &a1, float b0, float b1)
+{
+    asm("{\n\t.reg .b64 ra, rb;\n\t"
+        "mov.b64 ra, {%0, %1};\n\t"
+        "mov.b64 rb, {%2, %3};\n\t"
+        "add.rn.f32x2 ra, ra, rb;\n\t"
+        "mov.b64 {%0, %1}, ra;\n\t}"
+        : "+f"(a0), "+f"(a1)
+        : "f"(b0), "f"(b1));
+}
+
 // S_t = Q_t K^T: M = 128 query rows, N = 128 keys, K = D in steps of 16.
 // Both operands K-major, 128-byte swizzle, stored as D/64 blocks of
-// 128 rows x 128 bytes; 8-row groups are 1024 bytes apart.
+// 128 rows x 128 bytes; 8-row groups are 1024 bytes apart.  q_desc / k_desc
+// describe the tile bases; a k-step adds its byte offset / 16 to the start
+// address field (no carry: shared addresses stay below 256 KB).
 template <int D>
-__device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint32_t q_smem, uint32_t k_smem)
+__device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint64_t q_desc, uint64_t k_desc)
 {
     constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, BN, 0);
 #pragma unroll
     for (int kk = 0; kk < D / 16; ++kk) {
-        const uint32_t off = (kk >> 2) * Layout<D>::HALF_BYTES + (kk & 3) * 32;
-        ptx::mma_ss(s_tmem, ptx::smem_desc_sw128(q_smem + off, 16, 1024),
-                    ptx::smem_desc_sw128(k_smem + off, 16, 1024), idesc, kk > 0);
+        const uint32_t off = ((kk >> 2) * Layout<D>::HALF_BYTES + (kk & 3) * 32) >> 4;
+        ptx::mma_ss(s_tmem, q_desc + off, k_desc + off, idesc, kk > 0);
     }
 }
 
 // O_t (+)= P_t V: M = 128, N = D, K = 128 keys in steps of 16.  P comes from
 // TMEM (16 bf16 = 8 columns per step); V is N-major ("MN-major"): each key row
 // holds 64 contiguous head-dim values per 128-byte swizzled row, the two
-// 64-column blocks are HALF_BYTES apart (LBO), 8-key groups 1024 bytes (SBO).
+// 64-column blocks are HALF_BYTES apart (LBO), 8-key groups 1024 bytes (SBO);
+// a step of 16 keys advances 2048 bytes.
 template <int D>
-__device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint32_t v_smem, bool accumulate)
+__device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint64_t v_desc, bool accumulate)
 {
     constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, D, 1);
 #pragma unroll
-    for (int kk = 0; kk < BN / 16; ++kk) {
-        ptx::mma_ts(o_tmem, p_tmem + kk * 8, ptx::smem_desc_sw128(v_smem + kk * 2048, Layout<D>::HALF_BYTES, 1024),
-                    idesc, (accumulate || kk > 0) ? 1u : 0u);
-    }
+    for (int kk = 0; kk < BN / 16; ++kk)
+        ptx::mma_ts(o_tmem, p_tmem + kk * 8, v_desc + kk * (2048 >> 4), idesc, (accumulate || kk > 0) ? 1u : 0u);
 }
 
-// Row maximum (or minimum for a negative scale) of the raw logits, over the
-// first `valid` columns when PARTIAL.
+// Maximum (minimum for a negative scale) of the row's 128 raw logits; with
+// PARTIAL only the first `valid` of them count (valid >= 1).
 template <bool PARTIAL>
-__device__ __forceinline__ float tile_extreme(const uint32_t (&s)[4][32], bool neg_scale, int valid)
+__device__ __forceinline__ float row_extreme(const uint32_t (&s)[4][32], bool neg_scale, int valid)
 {
-    float e0 = neg_scale ? INFINITY : -INFINITY, e1 = e0, e2 = e0, e3 = e0;
+    const float pad = neg_scale ? INFINITY : -INFINITY;
+    float e0 = pad, e1 = pad, e2 = pad, e3 = pad;
 #pragma unroll
-    for (int c = 0; c < BN; c += 4) {
-        float x0 = __uint_as_float(s[c >> 5][c & 31]);
-        float x1 = __uint_as_float(s[c >> 5][(c & 31) + 1]);
-        float x2 = __uint_as_float(s[c >> 5][(c & 31) + 2]);
-        float x3 = __uint_as_float(s[c >> 5][(c & 31) + 3]);
-        if (PARTIAL) {
-            const float pad = neg_scale ? INFINITY : -INFINITY;
-            x0 = c + 0 < valid ? x0 : pad;
-            x1 = c + 1 < valid ? x1 : pad;
-            x2 = c + 2 < valid ? x2 : pad;
-            x3 = c + 3 < valid ? x3 : pad;
+    for (int c = 0; c < BN; c += 8) {
+        float x[8];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            x[i] = __uint_as_float(s[(c + i) >> 5][(c + i) & 31]);
+            if (PARTIAL)
+                x[i] = c + i < valid ? x[i] : pad;
         }
         if (neg_scale) {
-            e0 = fminf(e0, x0); e1 = fminf(e1, x1); e2 = fminf(e2, x2); e3 = fminf(e3, x3);
+            e0 = min3(e0, x[0], x[1]); e1 = min3(e1, x[2], x[3]);
+            e2 = min3(e2, x[4], x[5]); e3 = min3(e3, x[6], x[7]);
         } else {
-            e0 = fmaxf(e0, x0); e1 = fmaxf(e1, x1); e2 = fmaxf(e2, x2); e3 = fmaxf(e3, x3);
+            e0 = max3(e0, x[0], x[1]); e1 = max3(e1, x[2], x[3]);
+            e2 = max3(e2, x[4], x[5]); e3 = max3(e3, x[6], x[7]);
         }
     }
-    return neg_scale ? fminf(fminf(e0, e1), fminf(e2, e3)) : fmaxf(fmaxf(e0, e1), fmaxf(e2, e3));
+    return neg_scale ? min3(fminf(e0, e1), e2, e3) : max3(fmaxf(e0, e1), e2, e3);
 }
 
-// p = 2^(x * scale_log2 - m) for the 128 logits of this row, packed to bf16
-// pairs (even column in the low half); returns the fp32 sum of the p values.
+// p = 2^(x * scale_log2 - m) for the row's 128 logits, packed to bf16 pairs
+// (even key in the low half, 64 TMEM columns); returns the fp32 sum of p.
 template <bool PARTIAL>
-__device__ __forceinline__ float tile_probs(const uint32_t (&s)[4][32], uint32_t (&pk)[2][32], float sl2,
-                                            float neg_m, int valid)
+__device__ __forceinline__ float row_probs(const uint32_t (&s)[4][32], uint32_t (&pk)[2][32], float sl2,
+                                           float neg_m, int valid)
 {
     float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
     for (int c = 0; c < BN; c += 4) {
-        float p0 = ex2(fmaf(__uint_as_float(s[c >> 5][(c & 31) + 0]), sl2, neg_m));
-        float p1 = ex2(fmaf(__uint_as_float(s[c >> 5][(c & 31) + 1]), sl2, neg_m));
-        float p2 = ex2(fmaf(__uint_as_float(s[c >> 5][(c & 31) + 2]), sl2, neg_m));
-        float p3 = ex2(fmaf(__uint_as_float(s[c >> 5][(c & 31) + 3]), sl2, neg_m));
+        float x0, x1, x2, x3;
+        ffma2(x0, x1, __uint_as_float(s[c >> 5][(c & 31) + 0]), __uint_as_float(s[c >> 5][(c & 31) + 1]), sl2,
+              neg_m);
+        ffma2(x2, x3, __uint_as_float(s[c >> 5][(c & 31) + 2]), __uint_as_float(s[c >> 5][(c & 31) + 3]), sl2,
+              neg_m);
+        float p0 = ex2(x0), p1 = ex2(x1), p2 = ex2(x2), p3 = ex2(x3);
         if (PARTIAL) {
             p0 = c + 0 < valid ? p0 : 0.f;
             p1 = c + 1 < valid ? p1 : 0.f;
             p2 = c + 2 < valid ? p2 : 0.f;
             p3 = c + 3 < valid ? p3 : 0.f;
         }
-        a0 += p0;
-        a1 += p1;
-        a2 += p2;
-        a3 += p3;
+        fadd2(a0, a1, p0, p1);
+        fadd2(a2, a3, p2, p3);
         pk[c >> 6][(c & 63) >> 1] = pack_bf16x2(p0, p1);
         pk[c >> 6][((c & 63) >> 1) + 1] = pack_bf16x2(p2, p3);
     }
@@ -242,7 +293,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         for (int t = 0; t < 2; ++t) {
             ptx::mbar_init(bar(L::B_S + t), 1);
-            ptx::mbar_init(bar(L::B_P + t), 4 * 32);
+            ptx::mbar_init(bar(L::B_P + t), 4);   // one arrive per softmax warp
             ptx::mbar_init(bar(L::B_O + t), 1);
         }
         ptx::mbar_init(bar(L::B_FIX), 1);
@@ -325,10 +376,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     } else if (warp == MMA_WARP) {
         // ------------------------------------------------------------ tcgen05 issuer
         if (n_kv > 0 && lane == 0) {
-            const uint32_t q0 = sbase + L::Q_OFF;
-            const uint32_t q1 = q0 + L::TILE_BYTES;
+            // Shared-memory descriptors of the tile bases, computed once.
+            const uint64_t dq0 = ptx::smem_desc_sw128(sbase + L::Q_OFF, 16, 1024);
+            const uint64_t dq1 = ptx::smem_desc_sw128(sbase + L::Q_OFF + L::TILE_BYTES, 16, 1024);
+            const uint64_t dk = ptx::smem_desc_sw128(sbase + L::KV_OFF, 16, 1024);
+            const uint64_t dv = ptx::smem_desc_sw128(sbase + L::KV_OFF, L::HALF_BYTES, 1024);
+            constexpr uint32_t SLOT16 = L::TILE_BYTES >> 4;
             const uint32_t s0 = tmem, s1 = tmem + 128, o0 = tmem + 256, o1 = tmem + 384;
-            auto slot_addr = [&](int it) { return sbase + L::KV_OFF + (it % L::NSLOT) * L::TILE_BYTES; };
             auto full_wait = [&](int it) {
                 return wait_bounded(bar(L::B_FULL + it % L::NSLOT), (it / L::NSLOT) & 1, abort_flag, limit);
             };
@@ -336,37 +390,38 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                       wait_bounded(bar(L::B_Q + 1), 0, abort_flag, limit) && full_wait(0);
             if (ok) {
                 ptx::tc_fence_after_sync();
-                issue_qk<D>(s0, q0, slot_addr(0));
+                issue_qk<D>(s0, dq0, dk);
                 ptx::mma_commit(bar(L::B_S + 0));
-                issue_qk<D>(s1, q1, slot_addr(0));
+                issue_qk<D>(s1, dq1, dk);
                 ptx::mma_commit(bar(L::B_S + 1));
                 ptx::mma_commit(bar(L::B_EMPTY + 0));
-                for (int j = 0; j < n_kv && ok; ++j) {
+                for (int j = 0; j < n_kv; ++j) {
                     const int itv = 2 * j + 1, itk = 2 * j + 2;
                     const bool more = j + 1 < n_kv;
-                    ok = full_wait(itv) && wait_bounded(bar(L::B_P + 0), j & 1, abort_flag, limit);
-                    if (!ok)
+                    const uint64_t vd = dv + (itv % L::NSLOT) * SLOT16;
+                    const uint64_t kd = dk + (itk % L::NSLOT) * SLOT16;
+                    if (!(ok = full_wait(itv) && wait_bounded(bar(L::B_P + 0), j & 1, abort_flag, limit)))
                         break;
                     ptx::tc_fence_after_sync();
-                    issue_pv<D>(o0, s0, slot_addr(itv), j > 0);
+                    issue_pv<D>(o0, s0, vd, j > 0);
                     if (!more)
                         ptx::mma_commit(bar(L::B_O + 0));
                     if (more) {
                         if (!(ok = full_wait(itk)))
                             break;
                         ptx::tc_fence_after_sync();
-                        issue_qk<D>(s0, q0, slot_addr(itk));
+                        issue_qk<D>(s0, dq0, kd);
                         ptx::mma_commit(bar(L::B_S + 0));
                     }
                     if (!(ok = wait_bounded(bar(L::B_P + 1), j & 1, abort_flag, limit)))
                         break;
                     ptx::tc_fence_after_sync();
-                    issue_pv<D>(o1, s1, slot_addr(itv), j > 0);
+                    issue_pv<D>(o1, s1, vd, j > 0);
                     ptx::mma_commit(bar(L::B_EMPTY + itv % L::NSLOT));
                     if (!more)
                         ptx::mma_commit(bar(L::B_O + 1));
                     if (more) {
-                        issue_qk<D>(s1, q1, slot_addr(itk));
+                        issue_qk<D>(s1, dq1, kd);
                         ptx::mma_commit(bar(L::B_S + 1));
                         ptx::mma_commit(bar(L::B_EMPTY + itk % L::NSLOT));
                     }
@@ -384,7 +439,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         __syncwarp();
     } else {
-        // ------------------------------------------------------------ softmax groups
+        // ------------------------------------------------------------ softmax warps
         const int t = warp >> 2;                 // query tile of this group
         const int wq = warp & 3;                 // TMEM lane quarter of this warp
         const int q_row = (qp * 2 + t) * BM + wq * 32 + lane;
@@ -394,7 +449,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const float sl2 = p.scale_log2;
         const bool neg_scale = sl2 < 0.f;
         float m_used = -INFINITY;
-        float l = 0.f;
+        float l_exact = 0.f;   // sum of the fp32 weights: the log-sum-exp
+        float l_resid = 0.f;   // sum over tiles of r - p for each tile's largest weight
         bool ok = true;
 
         for (int j = 0; j < n_kv; ++j) {
@@ -409,7 +465,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
             const int valid = kv_valid - j * BN;
             const bool partial = valid < BN;
-            const float ext = partial ? tile_extreme<true>(s, neg_scale, valid) : tile_extreme<false>(s, neg_scale, BN);
+            const float ext = partial ? row_extreme<true>(s, neg_scale, valid) : row_extreme<false>(s, neg_scale, BN);
             const float m_tile = ext * sl2;
             const float m_new = fmaxf(m_used, m_tile);
             const bool need = m_new > m_used + TAU;
@@ -418,10 +474,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 factor = ex2(m_used - m_new);
                 m_used = m_new;
             }
-            l *= factor;
-            uint32_t pk[2][32];
             const float neg_m = -m_used;
-            l += partial ? tile_probs<true>(s, pk, sl2, neg_m, valid) : tile_probs<false>(s, pk, sl2, neg_m, BN);
+            // the tile's largest weight, computed exactly as in row_probs
+            const float p_top = ex2(fmaf(ext, sl2, neg_m));
+            l_exact *= factor;
+            l_resid = l_resid * factor + (round_bf16(p_top) - p_top);
+            uint32_t pk[2][32];
+            l_exact += partial ? row_probs<true>(s, pk, sl2, neg_m, valid) : row_probs<false>(s, pk, sl2, neg_m, BN);
             ptx::tmem_st32(s_addr, pk[0]);
             ptx::tmem_st32(s_addr + 32, pk[1]);
             if (j > 0 && __any_sync(0xffffffffu, need)) {
@@ -441,7 +500,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             ptx::tmem_wait_st();
             ptx::tc_fence_before_sync();
-            ptx::mbar_arrive(bar(L::B_P + t));
+            __syncwarp();
+            if (lane == 0)
+                ptx::mbar_arrive(bar(L::B_P + t));
         }
 
         // ------------------------------------------------------------ epilogue
@@ -457,7 +518,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
         } else if (ok && __all_sync(0xffffffffu, wait_bounded(bar(L::B_O + t), 0, abort_flag, limit))) {
             ptx::tc_fence_after_sync();
-            const float inv_l = 1.f / l;
+            const float inv_l = 1.f / (l_exact + l_resid);
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t r[32];
@@ -475,7 +536,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
             }
             if (store && p.lse)
-                p.lse[static_cast<size_t>(bh) * p.Sq + q_row] = (m_used + __log2f(l)) * 0.69314718055994530942f;
+                p.lse[static_cast<size_t>(bh) * p.Sq + q_row] = (m_used + __log2f(l_exact)) * 0.69314718055994530942f;
         }
     }
 
