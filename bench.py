@@ -255,15 +255,28 @@ def run_ours(args):
     print(json.dumps(line), flush=True)
 
 
+def kernel_source_hash():
+    """sha256 over the CUDA sources, to tell whether a stored ncu capture still applies."""
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_2609_18077_gb300", "csrc")
+    h = hashlib.sha256()
+    for name in sorted(os.listdir(csrc)):
+        if name.endswith((".cu", ".cuh", ".h")):
+            with open(os.path.join(csrc, name), "rb") as f:
+                h.update(name.encode() + b"\0" + f.read())
+    return h.hexdigest()[:16]
+
+
 def load_traffic(workload):
-    """DRAM bytes per launch from a committed ncu summary, when one matches the current kernel."""
+    """DRAM bytes per launch from the committed ncu summary, or None when the
+    kernel sources changed since that capture (or no capture covers the workload)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as f:
         d = json.load(f)
     entry = d.get(workload)
-    if not entry:
+    if not entry or entry.get("kernel_source_sha") != kernel_source_hash():
         return None
     return entry.get("dram_bytes_per_launch")
 
