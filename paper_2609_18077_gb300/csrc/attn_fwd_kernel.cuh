@@ -11,8 +11,9 @@
 // Work unit: one CTA owns one (b*h, pair of 128-row query tiles).  Roles:
 //   warps 0-3  softmax of query tile 0: thread = one query row (TMEM lane)
 //   warps 4-7  softmax of query tile 1
-//   warp  8    TMA producer: Q tiles once, then K_0 V_0 K_1 V_1 ... through a
-//              ring of NSLOT shared-memory slots
+//   warp  8    TMA producer: Q tiles once, then K_0 and the stages
+//              (V_0, K_1), (V_1, K_2), ... through a ring of NSTAGE
+//              two-tile stages (one full and one empty barrier per stage)
 //   warp  9    tcgen05 issuer (one lane) and TMEM owner
 // Tensor memory (512 columns x 128 lanes, fp32):
 //   S_t = cols [128t, 128t+128): logits Q_t K_j^T; the probabilities P_t are
@@ -22,6 +23,10 @@
 // MMA order per key tile j (ping-pong between the two query tiles so that the
 // softmax of one tile overlaps the GEMMs of the other):
 //   ... PV_0(j)  S_0(j+1)  PV_1(j)  S_1(j+1) ...
+// The issuing thread stalls on every barrier check (the tensor core holds
+// about one MMA ahead of execution), so it checks only P_t per step: the
+// softmax warps confirm that the step's V and next K have landed before they
+// publish P.
 // Online softmax in base 2 with a lazy maximum: a row's reference maximum m
 // only moves when the tile maximum exceeds it by more than TAU (log2 units),
 // so p <= 2^TAU and the O rescale in TMEM is rare after the first tiles.
@@ -76,15 +81,15 @@ struct Layout {
     static_assert(D == 64 || D == 128, "head dim");
     static constexpr int TILE_BYTES = BM * D * 2;           // one Q, K or V tile
     static constexpr int HALF_BYTES = BM * 128;              // one 64-column swizzle block
-    static constexpr int NSLOT = D == 128 ? 4 : 8;           // K/V ring
+    static constexpr int NSTAGE = D == 128 ? 2 : 4;          // K/V ring: stage = (V_j, K_{j+1})
     static constexpr int Q_OFF = 0;
-    static constexpr int KV_OFF = 2 * TILE_BYTES;
-    static constexpr int BAR_OFF = KV_OFF + NSLOT * TILE_BYTES;
+    static constexpr int KV_OFF = 2 * TILE_BYTES;            // stage s: V at 2s, K at 2s+1 (tiles)
+    static constexpr int BAR_OFF = KV_OFF + 2 * NSTAGE * TILE_BYTES;
     // barrier indices
     static constexpr int B_Q = 0;                            // [2] Q tile t landed
-    static constexpr int B_FULL = 2;                         // [NSLOT] slot landed
-    static constexpr int B_EMPTY = B_FULL + NSLOT;           // [NSLOT] slot consumed
-    static constexpr int B_S = B_EMPTY + NSLOT;              // [2] S_t ready
+    static constexpr int B_FULL = 2;                         // [NSTAGE] stage landed
+    static constexpr int B_EMPTY = B_FULL + NSTAGE;          // [NSTAGE] stage consumed
+    static constexpr int B_S = B_EMPTY + NSTAGE;             // [2] S_t ready
     static constexpr int B_P = B_S + 2;                      // [2] P_t written, O_t rescaled
     static constexpr int B_O = B_P + 2;                      // [2] last PV_t done
     static constexpr int B_FIX = B_O + 2;                    // varlen V tile staging
@@ -287,7 +292,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     if (threadIdx.x == 0) {
         ptx::mbar_init(bar(L::B_Q + 0), 1);
         ptx::mbar_init(bar(L::B_Q + 1), 1);
-        for (int i = 0; i < L::NSLOT; ++i) {
+        for (int i = 0; i < L::NSTAGE; ++i) {
             ptx::mbar_init(bar(L::B_FULL + i), 1);
             ptx::mbar_init(bar(L::B_EMPTY + i), 1);
         }
@@ -327,38 +332,45 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                          bar(L::B_Q + t), h * 64, (qp * 2 + t) * BM, bh);
                 }
             }
-            for (int it = 0; it < 2 * n_kv; ++it) {
-                const int slot = it % L::NSLOT;
-                if (it >= L::NSLOT) {
-                    if (!__all_sync(0xffffffffu,
-                                    wait_bounded(bar(L::B_EMPTY + slot), ((it / L::NSLOT) - 1) & 1, abort_flag, limit)))
-                        break;
-                }
-                const int j = it >> 1;
-                const bool is_v = it & 1;
-                const uint32_t dst = sbase + L::KV_OFF + slot * L::TILE_BYTES;
-                const CUtensorMap *tm = is_v ? &tmap_v : &tmap_k;
+            // Pair j >= 0 is the stage (V_j, K_{j+1}); pair -1 holds K_0 alone.
+            for (int j = -1; j < n_kv; ++j) {
+                const int st = (j + 1) % L::NSTAGE;
+                const int rnd = (j + 1) / L::NSTAGE;
+                if (rnd > 0 &&
+                    !__all_sync(0xffffffffu, wait_bounded(bar(L::B_EMPTY + st), (rnd - 1) & 1, abort_flag, limit)))
+                    break;
+                const bool has_v = j >= 0;
+                const bool has_k = j + 1 < n_kv;
                 const int valid_in_tile = kv_valid - j * BN;
-                if (!(VARLEN && is_v && valid_in_tile < BN)) {
+                const uint32_t vdst = sbase + L::KV_OFF + (2 * st) * L::TILE_BYTES;
+                const uint32_t kdst = vdst + L::TILE_BYTES;
+                if (!(VARLEN && has_v && valid_in_tile < BN)) {
                     if (lane == 0) {
-                        ptx::mbar_arrive_expect_tx(bar(L::B_FULL + slot), L::TILE_BYTES);
-                        for (int h = 0; h < D / 64; ++h)
-                            ptx::tma_load_3d(dst + h * L::HALF_BYTES, tm, bar(L::B_FULL + slot), h * 64, j * BN, bh);
+                        ptx::mbar_arrive_expect_tx(bar(L::B_FULL + st), (has_v + has_k) * L::TILE_BYTES);
+                        for (int h = 0; h < D / 64; ++h) {
+                            if (has_v)
+                                ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FULL + st), h * 64,
+                                                 j * BN, bh);
+                            if (has_k)
+                                ptx::tma_load_3d(kdst + h * L::HALF_BYTES, &tmap_k, bar(L::B_FULL + st), h * 64,
+                                                 (j + 1) * BN, bh);
+                        }
                     }
                 } else {
-                    // Last V tile of a padded sample: rows past the valid length
-                    // may hold any bits (NaN included) and 0 * NaN = NaN inside
-                    // the GEMM, so stage the tile, zero those rows, then publish.
+                    // Last V tile of a padded sample (no next K): rows past the
+                    // valid length may hold any bits (NaN included) and
+                    // 0 * NaN = NaN inside the GEMM, so stage the tile, zero
+                    // those rows, then publish the stage.
                     if (lane == 0) {
                         ptx::mbar_arrive_expect_tx(bar(L::B_FIX), L::TILE_BYTES);
                         for (int h = 0; h < D / 64; ++h)
-                            ptx::tma_load_3d(dst + h * L::HALF_BYTES, tm, bar(L::B_FIX), h * 64, j * BN, bh);
+                            ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FIX), h * 64, j * BN, bh);
                     }
                     if (!__all_sync(0xffffffffu, wait_bounded(bar(L::B_FIX), 0, abort_flag, limit)))
                         break;
                     const int nrow = BN - valid_in_tile;
                     const int per_half = nrow * 8;   // 16-byte chunks per 64-column block
-                    uint8_t *slot_ptr = sm + L::KV_OFF + slot * L::TILE_BYTES;
+                    uint8_t *slot_ptr = sm + L::KV_OFF + (2 * st) * L::TILE_BYTES;
                     for (int e = lane; e < per_half * (D / 64); e += 32) {
                         const int h = e / per_half;
                         const int rem = e - h * per_half;
@@ -369,7 +381,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     ptx::fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0)
-                        ptx::mbar_arrive(bar(L::B_FULL + slot));
+                        ptx::mbar_arrive(bar(L::B_FULL + st));
                 }
             }
         }
@@ -383,48 +395,44 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const uint64_t dv = ptx::smem_desc_sw128(sbase + L::KV_OFF, L::HALF_BYTES, 1024);
             constexpr uint32_t SLOT16 = L::TILE_BYTES >> 4;
             const uint32_t s0 = tmem, s1 = tmem + 128, o0 = tmem + 256, o1 = tmem + 384;
-            auto full_wait = [&](int it) {
-                return wait_bounded(bar(L::B_FULL + it % L::NSLOT), (it / L::NSLOT) & 1, abort_flag, limit);
-            };
+            // K_0 sits in the K slot of stage 0.
             bool ok = wait_bounded(bar(L::B_Q + 0), 0, abort_flag, limit) &&
-                      wait_bounded(bar(L::B_Q + 1), 0, abort_flag, limit) && full_wait(0);
+                      wait_bounded(bar(L::B_Q + 1), 0, abort_flag, limit) &&
+                      wait_bounded(bar(L::B_FULL + 0), 0, abort_flag, limit);
             if (ok) {
                 ptx::tc_fence_after_sync();
-                issue_qk<D>(s0, dq0, dk);
+                issue_qk<D>(s0, dq0, dk + SLOT16);
                 ptx::mma_commit(bar(L::B_S + 0));
-                issue_qk<D>(s1, dq1, dk);
+                issue_qk<D>(s1, dq1, dk + SLOT16);
                 ptx::mma_commit(bar(L::B_S + 1));
                 ptx::mma_commit(bar(L::B_EMPTY + 0));
                 for (int j = 0; j < n_kv; ++j) {
-                    const int itv = 2 * j + 1, itk = 2 * j + 2;
+                    // Stage (V_j, K_{j+1}); P_t(j) is published only after it landed.
+                    const int st = (j + 1) % L::NSTAGE;
+                    const uint64_t vd = dv + (2 * st) * SLOT16;
+                    const uint64_t kd = dk + (2 * st + 1) * SLOT16;
                     const bool more = j + 1 < n_kv;
-                    const uint64_t vd = dv + (itv % L::NSLOT) * SLOT16;
-                    const uint64_t kd = dk + (itk % L::NSLOT) * SLOT16;
-                    if (!(ok = full_wait(itv) && wait_bounded(bar(L::B_P + 0), j & 1, abort_flag, limit)))
+                    if (!(ok = wait_bounded(bar(L::B_P + 0), j & 1, abort_flag, limit)))
                         break;
                     ptx::tc_fence_after_sync();
                     issue_pv<D>(o0, s0, vd, j > 0);
-                    if (!more)
-                        ptx::mma_commit(bar(L::B_O + 0));
                     if (more) {
-                        if (!(ok = full_wait(itk)))
-                            break;
-                        ptx::tc_fence_after_sync();
                         issue_qk<D>(s0, dq0, kd);
                         ptx::mma_commit(bar(L::B_S + 0));
+                    } else {
+                        ptx::mma_commit(bar(L::B_O + 0));
                     }
                     if (!(ok = wait_bounded(bar(L::B_P + 1), j & 1, abort_flag, limit)))
                         break;
                     ptx::tc_fence_after_sync();
                     issue_pv<D>(o1, s1, vd, j > 0);
-                    ptx::mma_commit(bar(L::B_EMPTY + itv % L::NSLOT));
-                    if (!more)
-                        ptx::mma_commit(bar(L::B_O + 1));
                     if (more) {
                         issue_qk<D>(s1, dq1, kd);
                         ptx::mma_commit(bar(L::B_S + 1));
-                        ptx::mma_commit(bar(L::B_EMPTY + itk % L::NSLOT));
+                    } else {
+                        ptx::mma_commit(bar(L::B_O + 1));
                     }
+                    ptx::mma_commit(bar(L::B_EMPTY + st));
                 }
             }
             // Retire every MMA this thread issued before TMEM is released.
@@ -461,6 +469,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 #pragma unroll
             for (int c = 0; c < 4; ++c)
                 ptx::tmem_ld32(s_addr + 32 * c, s[c]);
+            // The stage (V_j, K_{j+1}) must have landed before P_t(j) is
+            // published; checked here, under the TMEM load latency.
+            if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + (j + 1) % L::NSTAGE),
+                                                            ((j + 1) / L::NSTAGE) & 1, abort_flag, limit)))) {
+                ptx::tmem_wait_ld();
+                break;
+            }
             ptx::tmem_wait_ld();
 
             const int valid = kv_valid - j * BN;
