@@ -8,7 +8,13 @@
 // sample's valid text length and masks the ragged last tile (appendix Table 4:
 // segment-id masking of padded text keys instead of a dense mask).
 //
-// Work unit: one CTA owns one (b*h, pair of 128-row query tiles).  Roles:
+// Work unit: one (b*h, pair of 128-row query tiles).  The grid is persistent:
+// one CTA per SM walks the units u = blockIdx.x, blockIdx.x + gridDim.x, ...
+// The K/V stream runs on across units (a unit's last stage carries the next
+// unit's K_0), each Q tile is reloaded as soon as the unit's last QK^T has
+// run, and each O accumulator is handed to the next unit as soon as the
+// epilogue holds it in registers, so one unit's start overlaps the previous
+// unit's end.  Roles:
 //   warps 0-3  softmax of query tile 0: thread = one query row (TMEM lane)
 //   warps 4-7  softmax of query tile 1
 //   warp  8    TMA producer: Q tiles once, then K_0 and the stages
@@ -72,6 +78,7 @@ struct AttnParams {
     int Sq;
     int Skv;              // Skv (dense) or Skv_max (varlen)
     int q_pairs;          // ceil(ceil(Sq / BM) / 2)
+    int units;            // B * H * q_pairs work units, handed out round-robin to the CTAs
     float scale_log2;     // scale * log2(e)
     uint64_t wait_limit_ns;
 };
@@ -87,12 +94,14 @@ struct Layout {
     static constexpr int BAR_OFF = KV_OFF + 2 * NSTAGE * TILE_BYTES;
     // barrier indices
     static constexpr int B_Q = 0;                            // [2] Q tile t landed
-    static constexpr int B_FULL = 2;                         // [NSTAGE] stage landed
+    static constexpr int B_QE = 2;                           // [2] Q tile t free (last QK^T of a unit ran)
+    static constexpr int B_FULL = 4;                         // [NSTAGE] stage landed
     static constexpr int B_EMPTY = B_FULL + NSTAGE;          // [NSTAGE] stage consumed
     static constexpr int B_S = B_EMPTY + NSTAGE;             // [2] S_t ready
     static constexpr int B_P = B_S + 2;                      // [2] P_t written, O_t rescaled
-    static constexpr int B_O = B_P + 2;                      // [2] last PV_t done
-    static constexpr int B_FIX = B_O + 2;                    // varlen V tile staging
+    static constexpr int B_O = B_P + 2;                      // [2] last PV_t of a unit done
+    static constexpr int B_OE = B_O + 2;                     // [2] O_t read out by the epilogue
+    static constexpr int B_FIX = B_OE + 2;                   // varlen V tile staging
     static constexpr int B_DRAIN = B_FIX + 1;                // all MMAs retired
     static constexpr int NBARS = B_DRAIN + 1;
     static constexpr int TMEM_PTR_OFF = BAR_OFF + NBARS * 8;
@@ -265,6 +274,29 @@ __device__ __forceinline__ float row_probs(const uint32_t (&s)[4][32], uint32_t 
     return (a0 + a1) + (a2 + a3);
 }
 
+// Per-unit geometry shared by every role: unit u = (b*h, pair of query tiles).
+struct Unit {
+    int bh;
+    int qp;
+    int kv_valid;
+    int n_kv;
+};
+
+template <bool VARLEN>
+__device__ __forceinline__ Unit unit_at(const AttnParams &p, int u)
+{
+    Unit w;
+    w.bh = u / p.q_pairs;
+    w.qp = u - w.bh * p.q_pairs;
+    w.kv_valid = p.Skv;
+    if (VARLEN) {
+        const int len = __ldg(p.kv_lens + w.bh / p.H);
+        w.kv_valid = len < 0 ? 0 : (len > p.Skv ? p.Skv : len);
+    }
+    w.n_kv = (w.kv_valid + BN - 1) / BN;
+    return w;
+}
+
 template <int D, bool VARLEN>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
@@ -277,29 +309,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     auto bar = [&](int i) -> uint32_t { return sbase + L::BAR_OFF + 8 * i; };
     volatile int *abort_flag = reinterpret_cast<volatile int *>(sm + L::ABORT_OFF);
     const uint64_t limit = p.wait_limit_ns;
-
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int bh = blockIdx.x / p.q_pairs;
-    const int qp = blockIdx.x - bh * p.q_pairs;
-    int kv_valid = p.Skv;
-    if (VARLEN) {
-        const int len = __ldg(p.kv_lens + bh / p.H);
-        kv_valid = len < 0 ? 0 : (len > p.Skv ? p.Skv : len);
-    }
-    const int n_kv = (kv_valid + BN - 1) / BN;
+    const int first_unit = blockIdx.x;
+    const int unit_step = gridDim.x;
 
     if (threadIdx.x == 0) {
-        ptx::mbar_init(bar(L::B_Q + 0), 1);
-        ptx::mbar_init(bar(L::B_Q + 1), 1);
+        for (int t = 0; t < 2; ++t) {
+            ptx::mbar_init(bar(L::B_Q + t), 1);
+            ptx::mbar_init(bar(L::B_QE + t), 1);
+            ptx::mbar_init(bar(L::B_S + t), 1);
+            ptx::mbar_init(bar(L::B_P + t), 4);    // one arrive per softmax warp
+            ptx::mbar_init(bar(L::B_O + t), 1);
+            ptx::mbar_init(bar(L::B_OE + t), 4);   // one arrive per softmax warp
+        }
         for (int i = 0; i < L::NSTAGE; ++i) {
             ptx::mbar_init(bar(L::B_FULL + i), 1);
             ptx::mbar_init(bar(L::B_EMPTY + i), 1);
-        }
-        for (int t = 0; t < 2; ++t) {
-            ptx::mbar_init(bar(L::B_S + t), 1);
-            ptx::mbar_init(bar(L::B_P + t), 4);   // one arrive per softmax warp
-            ptx::mbar_init(bar(L::B_O + t), 1);
         }
         ptx::mbar_init(bar(L::B_FIX), 1);
         ptx::mbar_init(bar(L::B_DRAIN), 1);
@@ -323,117 +349,178 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
     if (warp == PRODUCER_WARP) {
         // ------------------------------------------------------------ TMA producer
-        if (n_kv > 0) {
+        // Stage g of this CTA's stream holds (V_j, next K): j-th value tile of
+        // a unit and the key tile its GEMMs need next -- K_{j+1} of the same
+        // unit or K_0 of the next unit with keys.  Stage 0 holds K_0 alone.
+        auto next_with_keys = [&](int u) {
+            for (u += unit_step; u < p.units; u += unit_step)
+                if (unit_at<VARLEN>(p, u).n_kv > 0)
+                    return u;
+            return -1;
+        };
+        int g = 0;
+        int fixes = 0;
+        bool ok = true;
+        // load stage g: V tile (vbh, vj) if vj >= 0, K tile (kbh, kj) if kj >= 0
+        auto stage = [&](int vbh, int vj, int v_valid, int kbh, int kj) -> bool {
+            const int st = g % L::NSTAGE;
+            const int rnd = g / L::NSTAGE;
+            ++g;
+            if (rnd > 0 &&
+                !__all_sync(0xffffffffu, wait_bounded(bar(L::B_EMPTY + st), (rnd - 1) & 1, abort_flag, limit)))
+                return false;
+            const uint32_t vdst = sbase + L::KV_OFF + (2 * st) * L::TILE_BYTES;
+            const uint32_t kdst = vdst + L::TILE_BYTES;
+            const bool has_v = vj >= 0, has_k = kj >= 0;
+            const bool fix = VARLEN && has_v && v_valid < BN;
+            if (fix) {
+                // A padded sample's last V tile: rows past the valid length may
+                // hold any bits (NaN included) and 0 * NaN = NaN inside the
+                // GEMM, so stage the tile, zero those rows, then publish.
+                if (lane == 0) {
+                    ptx::mbar_arrive_expect_tx(bar(L::B_FIX), L::TILE_BYTES);
+                    for (int h = 0; h < D / 64; ++h)
+                        ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FIX), h * 64, vj * BN, vbh);
+                }
+                if (!__all_sync(0xffffffffu, wait_bounded(bar(L::B_FIX), fixes & 1, abort_flag, limit)))
+                    return false;
+                ++fixes;
+                const int per_half = (BN - v_valid) * 8;   // 16-byte chunks per 64-column block
+                uint8_t *slot_ptr = sm + L::KV_OFF + (2 * st) * L::TILE_BYTES;
+                for (int e = lane; e < per_half * (D / 64); e += 32) {
+                    const int h = e / per_half;
+                    const int rem = e - h * per_half;
+                    *reinterpret_cast<uint4 *>(slot_ptr + h * L::HALF_BYTES + (v_valid + (rem >> 3)) * 128 +
+                                               (rem & 7) * 16) = make_uint4(0u, 0u, 0u, 0u);
+                }
+                ptx::fence_proxy_async_smem();
+                __syncwarp();
+            }
+            if (lane == 0) {
+                const uint32_t bytes = ((has_v && !fix) + has_k) * L::TILE_BYTES;
+                if (bytes) {
+                    ptx::mbar_arrive_expect_tx(bar(L::B_FULL + st), bytes);
+                    for (int h = 0; h < D / 64; ++h) {
+                        if (has_v && !fix)
+                            ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FULL + st), h * 64,
+                                             vj * BN, vbh);
+                        if (has_k)
+                            ptx::tma_load_3d(kdst + h * L::HALF_BYTES, &tmap_k, bar(L::B_FULL + st), h * 64,
+                                             kj * BN, kbh);
+                    }
+                } else {
+                    ptx::mbar_arrive(bar(L::B_FULL + st));
+                }
+            }
+            return true;
+        };
+        int u = first_unit;
+        if (u < p.units && unit_at<VARLEN>(p, u).n_kv == 0)
+            u = next_with_keys(u);
+        if (u >= 0 && u < p.units)
+            ok = stage(0, -1, BN, unit_at<VARLEN>(p, u).bh, 0);
+        for (int iq = 0; ok && u >= 0 && u < p.units; ++iq) {
+            const Unit w = unit_at<VARLEN>(p, u);
+            const int nu = next_with_keys(u);
+            if (iq > 0) {
+                // Q tiles of the previous unit are free once its last QK^T ran.
+                ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_QE + 0), (iq - 1) & 1, abort_flag, limit) &&
+                                                 wait_bounded(bar(L::B_QE + 1), (iq - 1) & 1, abort_flag, limit));
+                if (!ok)
+                    break;
+            }
             if (lane == 0) {
                 for (int t = 0; t < 2; ++t) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_Q + t), L::TILE_BYTES);
                     for (int h = 0; h < D / 64; ++h)
                         ptx::tma_load_3d(sbase + L::Q_OFF + t * L::TILE_BYTES + h * L::HALF_BYTES, &tmap_q,
-                                         bar(L::B_Q + t), h * 64, (qp * 2 + t) * BM, bh);
+                                         bar(L::B_Q + t), h * 64, (w.qp * 2 + t) * BM, w.bh);
                 }
             }
-            // Pair j >= 0 is the stage (V_j, K_{j+1}); pair -1 holds K_0 alone.
-            for (int j = -1; j < n_kv; ++j) {
-                const int st = (j + 1) % L::NSTAGE;
-                const int rnd = (j + 1) / L::NSTAGE;
-                if (rnd > 0 &&
-                    !__all_sync(0xffffffffu, wait_bounded(bar(L::B_EMPTY + st), (rnd - 1) & 1, abort_flag, limit)))
-                    break;
-                const bool has_v = j >= 0;
-                const bool has_k = j + 1 < n_kv;
-                const int valid_in_tile = kv_valid - j * BN;
-                const uint32_t vdst = sbase + L::KV_OFF + (2 * st) * L::TILE_BYTES;
-                const uint32_t kdst = vdst + L::TILE_BYTES;
-                if (!(VARLEN && has_v && valid_in_tile < BN)) {
-                    if (lane == 0) {
-                        ptx::mbar_arrive_expect_tx(bar(L::B_FULL + st), (has_v + has_k) * L::TILE_BYTES);
-                        for (int h = 0; h < D / 64; ++h) {
-                            if (has_v)
-                                ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FULL + st), h * 64,
-                                                 j * BN, bh);
-                            if (has_k)
-                                ptx::tma_load_3d(kdst + h * L::HALF_BYTES, &tmap_k, bar(L::B_FULL + st), h * 64,
-                                                 (j + 1) * BN, bh);
-                        }
-                    }
-                } else {
-                    // Last V tile of a padded sample (no next K): rows past the
-                    // valid length may hold any bits (NaN included) and
-                    // 0 * NaN = NaN inside the GEMM, so stage the tile, zero
-                    // those rows, then publish the stage.
-                    if (lane == 0) {
-                        ptx::mbar_arrive_expect_tx(bar(L::B_FIX), L::TILE_BYTES);
-                        for (int h = 0; h < D / 64; ++h)
-                            ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FIX), h * 64, j * BN, bh);
-                    }
-                    if (!__all_sync(0xffffffffu, wait_bounded(bar(L::B_FIX), 0, abort_flag, limit)))
-                        break;
-                    const int nrow = BN - valid_in_tile;
-                    const int per_half = nrow * 8;   // 16-byte chunks per 64-column block
-                    uint8_t *slot_ptr = sm + L::KV_OFF + (2 * st) * L::TILE_BYTES;
-                    for (int e = lane; e < per_half * (D / 64); e += 32) {
-                        const int h = e / per_half;
-                        const int rem = e - h * per_half;
-                        const int r = valid_in_tile + (rem >> 3);
-                        *reinterpret_cast<uint4 *>(slot_ptr + h * L::HALF_BYTES + r * 128 + (rem & 7) * 16) =
-                            make_uint4(0u, 0u, 0u, 0u);
-                    }
-                    ptx::fence_proxy_async_smem();
-                    __syncwarp();
-                    if (lane == 0)
-                        ptx::mbar_arrive(bar(L::B_FULL + st));
-                }
+            for (int j = 0; ok && j < w.n_kv; ++j) {
+                const bool last = j + 1 == w.n_kv;
+                const int kbh = last ? (nu >= 0 ? unit_at<VARLEN>(p, nu).bh : 0) : w.bh;
+                const int kj = last ? (nu >= 0 ? 0 : -1) : j + 1;
+                ok = stage(w.bh, j, w.kv_valid - j * BN, kbh, kj);
             }
+            u = nu;
         }
     } else if (warp == MMA_WARP) {
         // ------------------------------------------------------------ tcgen05 issuer
-        if (n_kv > 0 && lane == 0) {
-            // Shared-memory descriptors of the tile bases, computed once.
+        if (lane == 0) {
             const uint64_t dq0 = ptx::smem_desc_sw128(sbase + L::Q_OFF, 16, 1024);
             const uint64_t dq1 = ptx::smem_desc_sw128(sbase + L::Q_OFF + L::TILE_BYTES, 16, 1024);
-            const uint64_t dk = ptx::smem_desc_sw128(sbase + L::KV_OFF, 16, 1024);
+            const uint64_t dk = ptx::smem_desc_sw128(sbase + L::KV_OFF + L::TILE_BYTES, 16, 1024);
             const uint64_t dv = ptx::smem_desc_sw128(sbase + L::KV_OFF, L::HALF_BYTES, 1024);
-            constexpr uint32_t SLOT16 = L::TILE_BYTES >> 4;
+            constexpr uint32_t STAGE16 = (2 * L::TILE_BYTES) >> 4;
             const uint32_t s0 = tmem, s1 = tmem + 128, o0 = tmem + 256, o1 = tmem + 384;
-            // K_0 sits in the K slot of stage 0.
-            bool ok = wait_bounded(bar(L::B_Q + 0), 0, abort_flag, limit) &&
-                      wait_bounded(bar(L::B_Q + 1), 0, abort_flag, limit) &&
-                      wait_bounded(bar(L::B_FULL + 0), 0, abort_flag, limit);
-            if (ok) {
+            int g = 1;         // stage holding (V_0, K_1) of the current unit
+            int pc = 0;        // P phases consumed (per tile, identical)
+            int iq = 0;        // units with keys so far
+            bool ok = true;
+            bool any = false;
+            for (int u = first_unit; ok && u < p.units; u += unit_step) {
+                const Unit w = unit_at<VARLEN>(p, u);
+                if (w.n_kv == 0)
+                    continue;
+                if (!any) {
+                    ok = wait_bounded(bar(L::B_FULL + 0), 0, abort_flag, limit);   // K_0 of the first unit
+                    any = true;
+                }
+                ok = ok && wait_bounded(bar(L::B_Q + 0), iq & 1, abort_flag, limit) &&
+                     wait_bounded(bar(L::B_Q + 1), iq & 1, abort_flag, limit);
+                if (!ok)
+                    break;
+                // K_0 sits in the stage before this unit's first.
+                const int st_k0 = (g - 1) % L::NSTAGE;
                 ptx::tc_fence_after_sync();
-                issue_qk<D>(s0, dq0, dk + SLOT16);
+                issue_qk<D>(s0, dq0, dk + st_k0 * STAGE16);
                 ptx::mma_commit(bar(L::B_S + 0));
-                issue_qk<D>(s1, dq1, dk + SLOT16);
+                issue_qk<D>(s1, dq1, dk + st_k0 * STAGE16);
                 ptx::mma_commit(bar(L::B_S + 1));
-                ptx::mma_commit(bar(L::B_EMPTY + 0));
-                for (int j = 0; j < n_kv; ++j) {
-                    // Stage (V_j, K_{j+1}); P_t(j) is published only after it landed.
-                    const int st = (j + 1) % L::NSTAGE;
-                    const uint64_t vd = dv + (2 * st) * SLOT16;
-                    const uint64_t kd = dk + (2 * st + 1) * SLOT16;
-                    const bool more = j + 1 < n_kv;
-                    if (!(ok = wait_bounded(bar(L::B_P + 0), j & 1, abort_flag, limit)))
+                // That stage also carried the previous unit's last V: both are done now.
+                ptx::mma_commit(bar(L::B_EMPTY + st_k0));
+                if (w.n_kv == 1) {
+                    ptx::mma_commit(bar(L::B_QE + 0));
+                    ptx::mma_commit(bar(L::B_QE + 1));
+                }
+                for (int j = 0; j < w.n_kv; ++j, ++pc) {
+                    const int st = (g + j) % L::NSTAGE;
+                    const uint64_t vd = dv + st * STAGE16;
+                    const uint64_t kd = dk + st * STAGE16;
+                    const bool more = j + 1 < w.n_kv;
+                    if (!(ok = wait_bounded(bar(L::B_P + 0), pc & 1, abort_flag, limit)))
+                        break;
+                    if (j == 0 && iq > 0 && !(ok = wait_bounded(bar(L::B_OE + 0), (iq - 1) & 1, abort_flag, limit)))
                         break;
                     ptx::tc_fence_after_sync();
                     issue_pv<D>(o0, s0, vd, j > 0);
                     if (more) {
                         issue_qk<D>(s0, dq0, kd);
                         ptx::mma_commit(bar(L::B_S + 0));
+                        if (j + 2 == w.n_kv)
+                            ptx::mma_commit(bar(L::B_QE + 0));
                     } else {
                         ptx::mma_commit(bar(L::B_O + 0));
                     }
-                    if (!(ok = wait_bounded(bar(L::B_P + 1), j & 1, abort_flag, limit)))
+                    if (!(ok = wait_bounded(bar(L::B_P + 1), pc & 1, abort_flag, limit)))
+                        break;
+                    if (j == 0 && iq > 0 && !(ok = wait_bounded(bar(L::B_OE + 1), (iq - 1) & 1, abort_flag, limit)))
                         break;
                     ptx::tc_fence_after_sync();
                     issue_pv<D>(o1, s1, vd, j > 0);
                     if (more) {
                         issue_qk<D>(s1, dq1, kd);
                         ptx::mma_commit(bar(L::B_S + 1));
+                        if (j + 2 == w.n_kv)
+                            ptx::mma_commit(bar(L::B_QE + 1));
+                        ptx::mma_commit(bar(L::B_EMPTY + st));
                     } else {
                         ptx::mma_commit(bar(L::B_O + 1));
                     }
-                    ptx::mma_commit(bar(L::B_EMPTY + st));
                 }
+                g += w.n_kv;
+                ++iq;
             }
             // Retire every MMA this thread issued before TMEM is released.
             ptx::mma_commit(bar(L::B_DRAIN));
@@ -450,108 +537,132 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // ------------------------------------------------------------ softmax warps
         const int t = warp >> 2;                 // query tile of this group
         const int wq = warp & 3;                 // TMEM lane quarter of this warp
-        const int q_row = (qp * 2 + t) * BM + wq * 32 + lane;
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>(wq * 32) << 16);
         const uint32_t s_addr = lane_addr + 128 * t;
         const uint32_t o_addr = lane_addr + 256 + 128 * t;
         const float sl2 = p.scale_log2;
         const bool neg_scale = sl2 < 0.f;
-        float m_used = -INFINITY;
-        float l_exact = 0.f;   // sum of the fp32 weights: the log-sum-exp
-        float l_resid = 0.f;   // sum over tiles of r - p for each tile's largest weight
+        int g = 1;      // stage of (V_0, K_1) of the current unit
+        int sc = 0;     // S phases consumed
+        int iq = 0;     // units with keys so far
         bool ok = true;
 
-        for (int j = 0; j < n_kv; ++j) {
-            if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_S + t), j & 1, abort_flag, limit))))
-                break;
-            ptx::tc_fence_after_sync();
-            uint32_t s[4][32];
+        for (int u = first_unit; ok && u < p.units; u += unit_step) {
+            const Unit w = unit_at<VARLEN>(p, u);
+            const int q_row = (w.qp * 2 + t) * BM + wq * 32 + lane;
+            const bool store = q_row < p.Sq;
+            __nv_bfloat16 *orow = p.out + (static_cast<size_t>(w.bh) * p.Sq + (store ? q_row : 0)) * D;
+            if (w.n_kv == 0) {
+                if (store) {
 #pragma unroll
-            for (int c = 0; c < 4; ++c)
-                ptx::tmem_ld32(s_addr + 32 * c, s[c]);
-            // The stage (V_j, K_{j+1}) must have landed before P_t(j) is
-            // published; checked here, under the TMEM load latency.
-            if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + (j + 1) % L::NSTAGE),
-                                                            ((j + 1) / L::NSTAGE) & 1, abort_flag, limit)))) {
-                ptx::tmem_wait_ld();
-                break;
-            }
-            ptx::tmem_wait_ld();
-
-            const int valid = kv_valid - j * BN;
-            const bool partial = valid < BN;
-            const float ext = partial ? row_extreme<true>(s, neg_scale, valid) : row_extreme<false>(s, neg_scale, BN);
-            const float m_tile = ext * sl2;
-            const float m_new = fmaxf(m_used, m_tile);
-            const bool need = m_new > m_used + TAU;
-            float factor = 1.f;
-            if (need) {
-                factor = ex2(m_used - m_new);
-                m_used = m_new;
-            }
-            const float neg_m = -m_used;
-            // the tile's largest weight, computed exactly as in row_probs
-            const float p_top = ex2(fmaf(ext, sl2, neg_m));
-            l_exact *= factor;
-            l_resid = l_resid * factor + (round_bf16(p_top) - p_top);
-            uint32_t pk[2][32];
-            l_exact += partial ? row_probs<true>(s, pk, sl2, neg_m, valid) : row_probs<false>(s, pk, sl2, neg_m, BN);
-            ptx::tmem_st32(s_addr, pk[0]);
-            ptx::tmem_st32(s_addr + 32, pk[1]);
-            if (j > 0 && __any_sync(0xffffffffu, need)) {
-                // O_t is idle here: S_t(j) was committed after PV_t(j-1), and
-                // PV_t(j) waits for the arrive below.  Done after P so that the
-                // logits' registers are free.
-#pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    uint32_t r[32];
-                    ptx::tmem_ld32(o_addr + 32 * c, r);
-                    ptx::tmem_wait_ld();
-#pragma unroll
-                    for (int i = 0; i < 32; ++i)
-                        r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
-                    ptx::tmem_st32(o_addr + 32 * c, r);
+                    for (int c = 0; c < D / 8; ++c)
+                        reinterpret_cast<uint4 *>(orow)[c] = make_uint4(0u, 0u, 0u, 0u);
+                    if (p.lse)
+                        p.lse[static_cast<size_t>(w.bh) * p.Sq + q_row] = -INFINITY;
                 }
+                continue;
             }
-            ptx::tmem_wait_st();
-            ptx::tc_fence_before_sync();
-            __syncwarp();
-            if (lane == 0)
-                ptx::mbar_arrive(bar(L::B_P + t));
-        }
-
-        // ------------------------------------------------------------ epilogue
-        const bool store = q_row < p.Sq;
-        __nv_bfloat16 *orow = p.out + (static_cast<size_t>(bh) * p.Sq + (store ? q_row : 0)) * D;
-        if (n_kv == 0) {
-            if (store) {
+            float m_used = -INFINITY;
+            float l_exact = 0.f;   // sum of the fp32 weights: the log-sum-exp
+            float l_resid = 0.f;   // sum over tiles of r - p for each tile's largest weight
+            for (int j = 0; j < w.n_kv; ++j, ++sc) {
+                if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_S + t), sc & 1, abort_flag, limit))))
+                    break;
+                ptx::tc_fence_after_sync();
+                uint32_t s[4][32];
 #pragma unroll
-                for (int c = 0; c < D / 8; ++c)
-                    reinterpret_cast<uint4 *>(orow)[c] = make_uint4(0u, 0u, 0u, 0u);
-                if (p.lse)
-                    p.lse[static_cast<size_t>(bh) * p.Sq + q_row] = -INFINITY;
+                for (int c = 0; c < 4; ++c)
+                    ptx::tmem_ld32(s_addr + 32 * c, s[c]);
+                // The stage (V_j, next K) must have landed before P_t(j) is
+                // published; checked here, under the TMEM load latency.
+                if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + (g + j) % L::NSTAGE),
+                                                                ((g + j) / L::NSTAGE) & 1, abort_flag, limit)))) {
+                    ptx::tmem_wait_ld();
+                    break;
+                }
+                ptx::tmem_wait_ld();
+
+                const int valid = w.kv_valid - j * BN;
+                const bool partial = valid < BN;
+                const float ext =
+                    partial ? row_extreme<true>(s, neg_scale, valid) : row_extreme<false>(s, neg_scale, BN);
+                const float m_tile = ext * sl2;
+                const float m_new = fmaxf(m_used, m_tile);
+                const bool need = m_new > m_used + TAU;
+                float factor = 1.f;
+                if (need) {
+                    factor = ex2(m_used - m_new);
+                    m_used = m_new;
+                }
+                const float neg_m = -m_used;
+                // the tile's largest weight, computed exactly as in row_probs
+                const float p_top = ex2(fmaf(ext, sl2, neg_m));
+                l_exact *= factor;
+                l_resid = l_resid * factor + (round_bf16(p_top) - p_top);
+                uint32_t pk[2][32];
+                l_exact +=
+                    partial ? row_probs<true>(s, pk, sl2, neg_m, valid) : row_probs<false>(s, pk, sl2, neg_m, BN);
+                ptx::tmem_st32(s_addr, pk[0]);
+                ptx::tmem_st32(s_addr + 32, pk[1]);
+                if (j > 0 && __any_sync(0xffffffffu, need)) {
+                    // O_t is idle here: S_t(j) was committed after PV_t(j-1), and
+                    // PV_t(j) waits for the arrive below.  Done after P so that the
+                    // logits' registers are free.
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint32_t r[32];
+                        ptx::tmem_ld32(o_addr + 32 * c, r);
+                        ptx::tmem_wait_ld();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
+                        ptx::tmem_st32(o_addr + 32 * c, r);
+                    }
+                }
+                ptx::tmem_wait_st();
+                ptx::tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0)
+                    ptx::mbar_arrive(bar(L::B_P + t));
             }
-        } else if (ok && __all_sync(0xffffffffu, wait_bounded(bar(L::B_O + t), 0, abort_flag, limit))) {
+            if (!ok)
+                break;
+
+            // -------------------------------------------------------- epilogue
+            if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_O + t), iq & 1, abort_flag, limit))))
+                break;
             ptx::tc_fence_after_sync();
             const float inv_l = 1.f / (l_exact + l_resid);
+            uint32_t w16[D / 32][16];
 #pragma unroll
             for (int c = 0; c < D / 32; ++c) {
                 uint32_t r[32];
                 ptx::tmem_ld32(o_addr + 32 * c, r);
                 ptx::tmem_wait_ld();
-                uint32_t w[16];
 #pragma unroll
                 for (int i = 0; i < 16; ++i)
-                    w[i] = pack_bf16x2(__uint_as_float(r[2 * i]) * inv_l, __uint_as_float(r[2 * i + 1]) * inv_l);
-                if (store) {
+                    w16[c][i] = pack_bf16x2(__uint_as_float(r[2 * i]) * inv_l, __uint_as_float(r[2 * i + 1]) * inv_l);
+            }
+            // O_t is in registers: hand the accumulator to the next unit's GEMMs
+            // before the global stores.
+            ptx::tc_fence_before_sync();
+            __syncwarp();
+            if (lane == 0)
+                ptx::mbar_arrive(bar(L::B_OE + t));
+            if (store) {
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
                     uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * c);
 #pragma unroll
                     for (int v = 0; v < 4; ++v)
-                        dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+                        dst[v] = make_uint4(w16[c][4 * v], w16[c][4 * v + 1], w16[c][4 * v + 2], w16[c][4 * v + 3]);
                 }
+                if (p.lse)
+                    p.lse[static_cast<size_t>(w.bh) * p.Sq + q_row] =
+                        (m_used + __log2f(l_exact)) * 0.69314718055994530942f;
             }
-            if (store && p.lse)
-                p.lse[static_cast<size_t>(bh) * p.Sq + q_row] = (m_used + __log2f(l_exact)) * 0.69314718055994530942f;
+            g += w.n_kv;
+            ++iq;
         }
     }
 

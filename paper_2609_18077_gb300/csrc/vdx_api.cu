@@ -43,6 +43,7 @@ EncodeTiledFn encode_fn()
 struct DeviceState {
     std::once_flag once;
     int status = VDX_OK;
+    int sms = 0;   // streaming multiprocessors: one persistent CTA each
 };
 DeviceState g_devices[kMaxDevices];
 
@@ -54,7 +55,8 @@ cudaError_t raise_smem_limit()
 }
 
 // One-time per-device check and kernel attribute set-up (current device).
-int device_ready()
+// Returns the status and, through *sms, the device's multiprocessor count.
+int device_ready(int *sms = nullptr)
 {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess)
@@ -73,6 +75,10 @@ int device_ready()
             st.status = VDX_ERR_DEVICE;
             return;
         }
+        if (cudaDeviceGetAttribute(&st.sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || st.sms <= 0) {
+            st.status = VDX_ERR_CUDA;
+            return;
+        }
         if (raise_smem_limit<64, false>() != cudaSuccess || raise_smem_limit<64, true>() != cudaSuccess ||
             raise_smem_limit<128, false>() != cudaSuccess || raise_smem_limit<128, true>() != cudaSuccess) {
             st.status = VDX_ERR_CUDA;
@@ -80,6 +86,8 @@ int device_ready()
         }
         st.status = encode_fn() ? VDX_OK : VDX_ERR_CUDA;
     });
+    if (sms)
+        *sms = st.sms;
     return st.status;
 }
 
@@ -136,7 +144,8 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         return VDX_ERR_INVALID_ARG;
 
     // ---- device set-up
-    int st = device_ready();
+    int sms = 0;
+    int st = device_ready(&sms);
     if (st != VDX_OK)
         return st;
 
@@ -154,10 +163,14 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     p.Sq = Sq;
     p.Skv = Skv;
     p.q_pairs = static_cast<int>(q_pairs);
+    p.units = static_cast<int>(bh * q_pairs);
     p.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
     p.wait_limit_ns = kWaitLimitNs;
 
-    const dim3 grid(static_cast<unsigned>(bh * q_pairs));
+    // Persistent grid: one CTA per multiprocessor (one fits per SM), each
+    // taking units blockIdx.x, blockIdx.x + grid, ... so that the CTAs
+    // running at any moment work on neighbouring units of the same heads.
+    const dim3 grid(static_cast<unsigned>(p.units < sms ? p.units : sms));
     const dim3 block(vdx::NUM_THREADS);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     if (D == 128) {

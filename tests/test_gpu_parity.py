@@ -126,3 +126,25 @@ def test_timeout_selftest_reports_and_recovers():
     assert binding.check_device_error() == binding.VDX_ERR_TIMEOUT
     assert binding.check_device_error() == binding.VDX_OK
     check_case(1, 1, 130, 140, 64, 0.125, seed=9)
+
+
+# More work units (b*h x query-tile pairs) than multiprocessors, so every
+# persistent CTA walks several units and the K/V stream crosses unit borders.
+MULTI_UNIT = [
+    # B, H, Sq, Skv, D
+    (1, 100, 300, 200, 128),
+    (2, 90, 513, 129, 64),
+    (3, 60, 256, 1, 128),
+]
+
+
+@pytest.mark.parametrize("B,H,Sq,Skv,D", MULTI_UNIT)
+def test_many_units_per_cta(B, H, Sq, Skv, D):
+    check_case(B, H, Sq, Skv, D, 1 / math.sqrt(D), seed=400 + H + Skv, gain=1.4)
+
+
+def test_varlen_many_units_mixed_lengths():
+    """Samples with no keys, one key, ragged and full tiles interleaved across
+    the units every CTA walks."""
+    lens = np.array([0, 300, 1, 129, 0, 256, 64, 255], np.int32)
+    check_case(8, 20, 257, 300, 128, 128 ** -0.5, seed=501, kv_lens=lens)
