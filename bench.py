@@ -59,6 +59,17 @@ def dist_env():
         int(os.environ.get("LOCAL_RANK", "0"))
 
 
+def max_over_ranks(x, world, device=None):
+    """Max of a host float over all ranks (identity for one rank); any backend."""
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle-reason sampling around the timed region."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
@@ -152,13 +163,6 @@ def run_ours(args):
             dist.barrier(device_ids=[local])
         torch.cuda.synchronize(dev)
 
-    def max_over_ranks(x):
-        if world == 1:
-            return x
-        t = torch.tensor([x], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        return float(t.item())
-
     for _ in range(args.warmup):
         step()
     st = binding.check_device_error(dev)
@@ -177,7 +181,7 @@ def run_ours(args):
             step()
         end.record(stream)
         barrier()
-    ms_total = max_over_ranks(start.elapsed_time(end))
+    ms_total = max_over_ranks(start.elapsed_time(end), world, dev)
     st = binding.check_device_error(dev)
     if st != binding.VDX_OK:
         raise RuntimeError(binding.status_string(st))
@@ -213,7 +217,7 @@ def run_ours(args):
         e2e_step()
     e2.record(stream)
     barrier()
-    e2e_ms = max_over_ranks(s2.elapsed_time(e2)) / e2e_steps
+    e2e_ms = max_over_ranks(s2.elapsed_time(e2), world, dev) / e2e_steps
     e2e_tflops = flops * world / (e2e_ms * 1e-3) / 1e12
 
     # ---- oracle on the host cores (rank 0, N = 1 only)
