@@ -79,7 +79,7 @@ struct AttnParams {
     int Skv;              // Skv (dense) or Skv_max (varlen)
     int q_pairs;          // ceil(ceil(Sq / BM) / 2)
     int units;            // B * H * q_pairs work units, handed out round-robin to the CTAs
-    float scale_log2;     // scale * log2(e)
+    float scale_log2;     // scale * log2(e); never 0: |value| >= 1e-30
     uint64_t wait_limit_ns;
 };
 
@@ -218,10 +218,8 @@ __device__ __forceinline__ void issue_pv(uint32_t o_tmem, uint32_t p_tmem, uint6
         ptx::mma_ts(o_tmem, p_tmem + kk * 8, v_desc + kk * (2048 >> 4), idesc, (accumulate || kk > 0) ? 1u : 0u);
 }
 
-// Maximum (minimum for a negative scale) of the row's 128 raw logits; with
-// PARTIAL only the first `valid` of them count (valid >= 1).
-template <bool PARTIAL>
-__device__ __forceinline__ float row_extreme(const uint32_t (&s)[4][32], bool neg_scale, int valid)
+// Maximum (minimum for a negative scale) of the row's 128 raw logits.
+__device__ __forceinline__ float row_extreme(const uint32_t (&s)[4][32], bool neg_scale)
 {
     const float pad = neg_scale ? INFINITY : -INFINITY;
     float e0 = pad, e1 = pad, e2 = pad, e3 = pad;
@@ -229,11 +227,8 @@ __device__ __forceinline__ float row_extreme(const uint32_t (&s)[4][32], bool ne
     for (int c = 0; c < BN; c += 8) {
         float x[8];
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
+        for (int i = 0; i < 8; ++i)
             x[i] = __uint_as_float(s[(c + i) >> 5][(c + i) & 31]);
-            if (PARTIAL)
-                x[i] = c + i < valid ? x[i] : pad;
-        }
         if (neg_scale) {
             e0 = min3(e0, x[0], x[1]); e1 = min3(e1, x[2], x[3]);
             e2 = min3(e2, x[4], x[5]); e3 = min3(e3, x[6], x[7]);
@@ -247,9 +242,7 @@ __device__ __forceinline__ float row_extreme(const uint32_t (&s)[4][32], bool ne
 
 // p = 2^(x * scale_log2 - m) for the row's 128 logits, packed to bf16 pairs
 // (even key in the low half, 64 TMEM columns); returns the fp32 sum of p.
-template <bool PARTIAL>
-__device__ __forceinline__ float row_probs(const uint32_t (&s)[4][32], uint32_t (&pk)[2][32], float sl2,
-                                           float neg_m, int valid)
+__device__ __forceinline__ float row_probs(const uint32_t (&s)[4][32], uint32_t (&pk)[2][32], float sl2, float neg_m)
 {
     float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
@@ -259,13 +252,7 @@ __device__ __forceinline__ float row_probs(const uint32_t (&s)[4][32], uint32_t 
               neg_m);
         ffma2(x2, x3, __uint_as_float(s[c >> 5][(c & 31) + 2]), __uint_as_float(s[c >> 5][(c & 31) + 3]), sl2,
               neg_m);
-        float p0 = ex2(x0), p1 = ex2(x1), p2 = ex2(x2), p3 = ex2(x3);
-        if (PARTIAL) {
-            p0 = c + 0 < valid ? p0 : 0.f;
-            p1 = c + 1 < valid ? p1 : 0.f;
-            p2 = c + 2 < valid ? p2 : 0.f;
-            p3 = c + 3 < valid ? p3 : 0.f;
-        }
+        const float p0 = ex2(x0), p1 = ex2(x1), p2 = ex2(x2), p3 = ex2(x3);
         fadd2(a0, a1, p0, p1);
         fadd2(a2, a3, p2, p3);
         pk[c >> 6][(c & 63) >> 1] = pack_bf16x2(p0, p1);
@@ -583,9 +570,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 ptx::tmem_wait_ld();
 
                 const int valid = w.kv_valid - j * BN;
-                const bool partial = valid < BN;
-                const float ext =
-                    partial ? row_extreme<true>(s, neg_scale, valid) : row_extreme<false>(s, neg_scale, BN);
+                if (valid < BN) {
+                    // Ragged last tile: keys past the end (or past the sample's
+                    // text length, whatever their bits) become -inf logits
+                    // after scaling, i.e. weight exactly 0.  scale_log2 is never
+                    // 0 (the host raises it to 1e-30), so inf * scale stays inf.
+                    const uint32_t pad = neg_scale ? 0x7F800000u : 0xFF800000u;
+#pragma unroll
+                    for (int c = 0; c < BN; ++c)
+                        s[c >> 5][c & 31] = c < valid ? s[c >> 5][c & 31] : pad;
+                }
+                const float ext = row_extreme(s, neg_scale);
                 const float m_tile = ext * sl2;
                 const float m_new = fmaxf(m_used, m_tile);
                 const bool need = m_new > m_used + TAU;
@@ -600,8 +595,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 l_exact *= factor;
                 l_resid = l_resid * factor + (round_bf16(p_top) - p_top);
                 uint32_t pk[2][32];
-                l_exact +=
-                    partial ? row_probs<true>(s, pk, sl2, neg_m, valid) : row_probs<false>(s, pk, sl2, neg_m, BN);
+                l_exact += row_probs(s, pk, sl2, neg_m);
                 ptx::tmem_st32(s_addr, pk[0]);
                 ptx::tmem_st32(s_addr + 32, pk[1]);
                 if (j > 0 && __any_sync(0xffffffffu, need)) {

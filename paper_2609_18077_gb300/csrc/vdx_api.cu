@@ -164,7 +164,13 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     p.Skv = Skv;
     p.q_pairs = static_cast<int>(q_pairs);
     p.units = static_cast<int>(bh * q_pairs);
-    p.scale_log2 = static_cast<float>(static_cast<double>(scale) * 1.4426950408889634074);
+    // A zero (or tinier than 1e-30) logit scale is raised to 1e-30: every
+    // weight is then still exactly 1 for finite logits, and masked keys
+    // (+-inf logits) keep weight 0 instead of inf * 0 = NaN.
+    double sl2 = static_cast<double>(scale) * 1.4426950408889634074;
+    if (std::fabs(sl2) < 1e-30)
+        sl2 = sl2 < 0 ? -1e-30 : 1e-30;
+    p.scale_log2 = static_cast<float>(sl2);
     p.wait_limit_ns = kWaitLimitNs;
 
     // Persistent grid: one CTA per multiprocessor (one fits per SM), each
