@@ -79,6 +79,7 @@ struct AttnParams {
     int Skv;              // Skv (dense) or Skv_max (varlen)
     int q_pairs;          // ceil(ceil(Sq / BM) / 2)
     int units;            // B * H * q_pairs work units, handed out round-robin to the CTAs
+    int out_align32;      // out is 32-byte aligned: write O with 256-bit stores
     float scale_log2;     // scale * log2(e); never 0: |value| >= 1e-30
     uint64_t wait_limit_ns;
 };
@@ -644,12 +645,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             if (lane == 0)
                 ptx::mbar_arrive(bar(L::B_OE + t));
             if (store) {
+                if (p.out_align32) {
+                    // 32-byte stores: each fills a whole sector of the row.
 #pragma unroll
-                for (int c = 0; c < D / 32; ++c) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * c);
+                    for (int c = 0; c < D / 32; ++c)
 #pragma unroll
-                    for (int v = 0; v < 4; ++v)
-                        dst[v] = make_uint4(w16[c][4 * v], w16[c][4 * v + 1], w16[c][4 * v + 2], w16[c][4 * v + 3]);
+                        for (int v = 0; v < 2; ++v)
+                            ptx::st_global_v8(orow + 32 * c + 16 * v, &w16[c][8 * v]);
+                } else {
+#pragma unroll
+                    for (int c = 0; c < D / 32; ++c) {
+                        uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * c);
+#pragma unroll
+                        for (int v = 0; v < 4; ++v)
+                            dst[v] = make_uint4(w16[c][4 * v], w16[c][4 * v + 1], w16[c][4 * v + 2], w16[c][4 * v + 3]);
+                    }
                 }
                 if (p.lse)
                     p.lse[static_cast<size_t>(w.bh) * p.Sq + q_row] =

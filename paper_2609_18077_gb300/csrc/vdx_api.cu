@@ -164,6 +164,7 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     p.Skv = Skv;
     p.q_pairs = static_cast<int>(q_pairs);
     p.units = static_cast<int>(bh * q_pairs);
+    p.out_align32 = aligned(out, 32) ? 1 : 0;
     // A zero (or tinier than 1e-30) logit scale is raised to 1e-30: every
     // weight is then still exactly 1 for finite logits, and masked keys
     // (+-inf logits) keep weight 0 instead of inf * 0 = NaN.
