@@ -22,8 +22,16 @@
  *   - Tensors are contiguous, row-major, bf16 (IEEE bfloat16 bits):
  *       q, out: [B, H, Sq, D];  k, v: [B, H, Skv, D];  lse: fp32 [B, H, Sq].
  *   - All tensor pointers are DEVICE pointers owned by the caller; the
- *     library never frees or keeps them after the call returns, and it
- *     allocates no device memory per call.
+ *     library never frees or keeps them after the call returns.
+ *   - Memory: when the last round of work units would leave most
+ *     multiprocessors idle (dense calls only), the library splits those units
+ *     along the keys and merges the parts through a device workspace of
+ *     (tail units x parts x 2 x 128 x (D + 4)) fp32 values -- about 19 MB for
+ *     B=1, H=12, S=32760, D=128.  The workspace belongs to the library, one per
+ *     (device, stream): it is allocated by the first call that needs it, grown
+ *     by a later call that needs more (that call waits for the device), and
+ *     kept until the process exits.  Calls on the same stream share it in
+ *     stream order; calls on different streams never share it.
  *   - q, k, v and out must be 16-byte aligned (TMA and vector stores); lse
  *     4-byte aligned.  out must not overlap q, k or v.
  *   - D must be 64 or 128.  B, H, Sq, Skv >= 0; B*H*Sq == 0 is a no-op.

@@ -80,6 +80,15 @@ struct AttnParams {
     int q_pairs;          // ceil(ceil(Sq / BM) / 2)
     int units;            // B * H * q_pairs work units, handed out round-robin to the CTAs
     int out_align32;      // out is 32-byte aligned: write O with 256-bit stores
+    // Split tail (0 parts: off).  The first full_rounds * gridDim.x units are
+    // whole items; each of the tail_units remaining ones is cut into
+    // split_parts key ranges, one per CTA, merged through the workspace.
+    int split_parts;
+    int full_rounds;
+    int tail_units;
+    float *ws_o;          // [tail_units][split_parts][2][BM][D] unnormalised fp32 accumulators
+    float *ws_stats;      // [tail_units][split_parts][2][BM] float4 (m, l_exact, l_resid, -)
+    int *ws_count;        // [tail_units] parts finished (zeroed before the launch)
     float scale_log2;     // scale * log2(e); never 0: |value| >= 1e-30
     uint64_t wait_limit_ns;
 };
@@ -104,10 +113,12 @@ struct Layout {
     static constexpr int B_OE = B_O + 2;                     // [2] O_t read out by the epilogue
     static constexpr int B_FIX = B_OE + 2;                   // varlen V tile staging
     static constexpr int B_DRAIN = B_FIX + 1;                // all MMAs retired
-    static constexpr int NBARS = B_DRAIN + 1;
+    static constexpr int B_MERGE = B_DRAIN + 1;              // [2] tail part written (8 warps) / merge decided
+    static constexpr int NBARS = B_MERGE + 2;
     static constexpr int TMEM_PTR_OFF = BAR_OFF + NBARS * 8;
     static constexpr int ABORT_OFF = TMEM_PTR_OFF + 4;
-    static constexpr int BYTES = ABORT_OFF + 4;
+    static constexpr int MERGE_OFF = ABORT_OFF + 4;          // "this CTA merges" flag
+    static constexpr int BYTES = MERGE_OFF + 4;
     static constexpr int ALLOC = BYTES + 1024;               // slack for 1024-B alignment
 };
 
@@ -262,18 +273,99 @@ __device__ __forceinline__ float row_probs(const uint32_t (&s)[4][32], uint32_t 
     return (a0 + a1) + (a2 + a3);
 }
 
-// Per-unit geometry shared by every role: unit u = (b*h, pair of query tiles).
-struct Unit {
+// Merge of a split tail unit, run by the CTA that finishes its last part.
+// Every part wrote, per query row, its unnormalised fp32 accumulator O_k and
+// (m_k, le_k, lr_k): running maximum (log2 units), exact weight sum and
+// rounding-residual sum.  With M = max m_k and w_k = 2^(m_k - M):
+//   O = sum_k w_k O_k / sum_k w_k (le_k + lr_k),  LSE = (M + log2 sum_k w_k le_k) ln 2.
+template <int D>
+__device__ __noinline__ void merge_tail_parts(const AttnParams &p, int tail, int t, int row, int q_row, int bh,
+                                              bool store, __nv_bfloat16 *orow, volatile int *last_flag,
+                                              uint32_t bar_written, uint32_t bar_decided, volatile int *abort_flag)
+{
+    // All eight softmax warps wrote their rows of the part; publish them.  The
+    // two waits are bounded, so a CTA that aborted elsewhere cannot hang here.
+    const int lane = threadIdx.x & 31;
+    __threadfence();
+    __syncwarp();
+    if (lane == 0)
+        ptx::mbar_arrive(bar_written);
+    if (threadIdx.x == 0) {
+        int last = 0;
+        if (wait_bounded(bar_written, 0, abort_flag, p.wait_limit_ns)) {
+            const int done = atomicAdd(p.ws_count + tail, 1);
+            last = done == p.split_parts - 1;
+        }
+        *last_flag = last;
+        ptx::mbar_arrive(bar_decided);
+    }
+    if (!__all_sync(0xffffffffu, wait_bounded(bar_decided, 0, abort_flag, p.wait_limit_ns)) || !*last_flag)
+        return;
+    __threadfence();
+    const int P = p.split_parts;
+    auto slot = [&](int k) { return (tail * P + k) * 2 + t; };
+    float M = -INFINITY;
+    for (int k = 0; k < P; ++k)
+        M = fmaxf(M, __ldcg(reinterpret_cast<const float4 *>(p.ws_stats) + slot(k) * BM + row).x);
+    float le = 0.f, lc = 0.f;
+    for (int k = 0; k < P; ++k) {
+        const float4 st = __ldcg(reinterpret_cast<const float4 *>(p.ws_stats) + slot(k) * BM + row);
+        const float wk = ex2(st.x - M);
+        le += wk * st.y;
+        lc += wk * (st.y + st.z);
+    }
+    const float inv = 1.f / lc;
+#pragma unroll
+    for (int c = 0; c < D / 32; ++c) {
+        float acc[32];
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+            acc[i] = 0.f;
+        for (int k = 0; k < P; ++k) {
+            const float wk = ex2(__ldcg(reinterpret_cast<const float4 *>(p.ws_stats) + slot(k) * BM + row).x - M);
+            const float4 *src = reinterpret_cast<const float4 *>(p.ws_o + (static_cast<size_t>(slot(k)) * BM + row) * D +
+                                                                 32 * c);
+#pragma unroll
+            for (int v = 0; v < 8; ++v) {
+                const float4 x = __ldcg(src + v);
+                acc[4 * v + 0] = fmaf(wk, x.x, acc[4 * v + 0]);
+                acc[4 * v + 1] = fmaf(wk, x.y, acc[4 * v + 1]);
+                acc[4 * v + 2] = fmaf(wk, x.z, acc[4 * v + 2]);
+                acc[4 * v + 3] = fmaf(wk, x.w, acc[4 * v + 3]);
+            }
+        }
+        if (store) {
+            uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+                dst[v] = make_uint4(pack_bf16x2(acc[8 * v] * inv, acc[8 * v + 1] * inv),
+                                    pack_bf16x2(acc[8 * v + 2] * inv, acc[8 * v + 3] * inv),
+                                    pack_bf16x2(acc[8 * v + 4] * inv, acc[8 * v + 5] * inv),
+                                    pack_bf16x2(acc[8 * v + 6] * inv, acc[8 * v + 7] * inv));
+        }
+    }
+    if (store && p.lse)
+        p.lse[static_cast<size_t>(bh) * p.Sq + q_row] = (M + __log2f(le)) * 0.69314718055994530942f;
+}
+
+// One work item of a CTA: a whole unit (b*h, query-tile pair) with key tiles
+// [j0, j1) = [0, n_kv), or -- for the units of a short last round, when the
+// host splits them -- one part of such a unit's key tiles (part >= 0).
+struct Item {
     int bh;
     int qp;
     int kv_valid;
-    int n_kv;
+    int n_kv;      // key tiles of the whole unit
+    int j0, j1;    // key tiles of this item
+    int part;      // -1: whole unit; else the part index within tail unit `tail`
+    int tail;
+    bool ok;       // false past the CTA's last item
 };
 
 template <bool VARLEN>
-__device__ __forceinline__ Unit unit_at(const AttnParams &p, int u)
+__device__ __forceinline__ Item unit_item(const AttnParams &p, int u)
 {
-    Unit w;
+    Item w;
     w.bh = u / p.q_pairs;
     w.qp = u - w.bh * p.q_pairs;
     w.kv_valid = p.Skv;
@@ -282,6 +374,39 @@ __device__ __forceinline__ Unit unit_at(const AttnParams &p, int u)
         w.kv_valid = len < 0 ? 0 : (len > p.Skv ? p.Skv : len);
     }
     w.n_kv = (w.kv_valid + BN - 1) / BN;
+    w.j0 = 0;
+    w.j1 = w.n_kv;
+    w.part = -1;
+    w.tail = 0;
+    w.ok = true;
+    return w;
+}
+
+// The i-th item of CTA `cta`: units cta, cta + G, ... and, in split mode,
+// after full_rounds of them one part of a tail unit.
+template <bool VARLEN>
+__device__ __forceinline__ Item item_at(const AttnParams &p, int cta, int i)
+{
+    const int G = gridDim.x;
+    Item w;
+    w.ok = false;
+    if (p.split_parts == 0) {
+        const int u = cta + i * G;
+        if (u < p.units)
+            w = unit_item<VARLEN>(p, u);
+        return w;
+    }
+    if (i < p.full_rounds)
+        return unit_item<VARLEN>(p, cta + i * G);
+    if (i == p.full_rounds && cta < p.tail_units * p.split_parts) {
+        const int tail = cta / p.split_parts;
+        const int part = cta - tail * p.split_parts;
+        w = unit_item<VARLEN>(p, p.full_rounds * G + tail);
+        w.j0 = part * w.n_kv / p.split_parts;
+        w.j1 = (part + 1) * w.n_kv / p.split_parts;
+        w.part = part;
+        w.tail = tail;
+    }
     return w;
 }
 
@@ -299,8 +424,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const uint64_t limit = p.wait_limit_ns;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int first_unit = blockIdx.x;
-    const int unit_step = gridDim.x;
+    const int cta = blockIdx.x;
 
     if (threadIdx.x == 0) {
         for (int t = 0; t < 2; ++t) {
@@ -317,6 +441,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         ptx::mbar_init(bar(L::B_FIX), 1);
         ptx::mbar_init(bar(L::B_DRAIN), 1);
+        ptx::mbar_init(bar(L::B_MERGE + 0), 8);
+        ptx::mbar_init(bar(L::B_MERGE + 1), 1);
         *abort_flag = 0;
         ptx::fence_barrier_init();
         ptx::fence_proxy_async_smem();
@@ -337,14 +463,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
     if (warp == PRODUCER_WARP) {
         // ------------------------------------------------------------ TMA producer
-        // Stage g of this CTA's stream holds (V_j, next K): j-th value tile of
-        // a unit and the key tile its GEMMs need next -- K_{j+1} of the same
-        // unit or K_0 of the next unit with keys.  Stage 0 holds K_0 alone.
-        auto next_with_keys = [&](int u) {
-            for (u += unit_step; u < p.units; u += unit_step)
-                if (unit_at<VARLEN>(p, u).n_kv > 0)
-                    return u;
-            return -1;
+        // Stage g of this CTA's stream holds (V_j, next K): the j-th value tile
+        // of an item and the key tile its GEMMs need next -- K_{j+1} of the
+        // same item or the first key tile of the next item with keys.  Stage 0
+        // holds that first key tile alone.
+        auto next_with_keys = [&](int i) {
+            for (++i;; ++i) {
+                const Item w = item_at<VARLEN>(p, cta, i);
+                if (!w.ok)
+                    return -1;
+                if (w.j1 > w.j0)
+                    return i;
+            }
         };
         int g = 0;
         int fixes = 0;
@@ -402,16 +532,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             return true;
         };
-        int u = first_unit;
-        if (u < p.units && unit_at<VARLEN>(p, u).n_kv == 0)
-            u = next_with_keys(u);
-        if (u >= 0 && u < p.units)
-            ok = stage(0, -1, BN, unit_at<VARLEN>(p, u).bh, 0);
-        for (int iq = 0; ok && u >= 0 && u < p.units; ++iq) {
-            const Unit w = unit_at<VARLEN>(p, u);
-            const int nu = next_with_keys(u);
+        int i = 0;
+        {
+            const Item w0 = item_at<VARLEN>(p, cta, 0);
+            if (!w0.ok)
+                i = -1;
+            else if (w0.j1 == w0.j0)
+                i = next_with_keys(0);
+        }
+        if (i >= 0) {
+            const Item w = item_at<VARLEN>(p, cta, i);
+            ok = stage(0, -1, BN, w.bh, w.j0);
+        }
+        for (int iq = 0; ok && i >= 0; ++iq) {
+            const Item w = item_at<VARLEN>(p, cta, i);
+            const int ni = next_with_keys(i);
             if (iq > 0) {
-                // Q tiles of the previous unit are free once its last QK^T ran.
+                // Q tiles of the previous item are free once its last QK^T ran.
                 ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_QE + 0), (iq - 1) & 1, abort_flag, limit) &&
                                                  wait_bounded(bar(L::B_QE + 1), (iq - 1) & 1, abort_flag, limit));
                 if (!ok)
@@ -425,13 +562,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                          bar(L::B_Q + t), h * 64, (w.qp * 2 + t) * BM, w.bh);
                 }
             }
-            for (int j = 0; ok && j < w.n_kv; ++j) {
-                const bool last = j + 1 == w.n_kv;
-                const int kbh = last ? (nu >= 0 ? unit_at<VARLEN>(p, nu).bh : 0) : w.bh;
-                const int kj = last ? (nu >= 0 ? 0 : -1) : j + 1;
+            Item nw;
+            nw.ok = false;
+            if (ni >= 0)
+                nw = item_at<VARLEN>(p, cta, ni);
+            for (int j = w.j0; ok && j < w.j1; ++j) {
+                const bool last = j + 1 == w.j1;
+                const int kbh = last ? (nw.ok ? nw.bh : 0) : w.bh;
+                const int kj = last ? (nw.ok ? nw.j0 : -1) : j + 1;
                 ok = stage(w.bh, j, w.kv_valid - j * BN, kbh, kj);
             }
-            u = nu;
+            i = ni;
         }
     } else if (warp == MMA_WARP) {
         // ------------------------------------------------------------ tcgen05 issuer
@@ -442,72 +583,72 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const uint64_t dv = ptx::smem_desc_sw128(sbase + L::KV_OFF, L::HALF_BYTES, 1024);
             constexpr uint32_t STAGE16 = (2 * L::TILE_BYTES) >> 4;
             const uint32_t s0 = tmem, s1 = tmem + 128, o0 = tmem + 256, o1 = tmem + 384;
-            int g = 1;         // stage holding (V_0, K_1) of the current unit
+            int g = 1;         // stage holding the current item's (V_j0, next K)
             int pc = 0;        // P phases consumed (per tile, identical)
-            int iq = 0;        // units with keys so far
+            int iq = 0;        // items with keys so far
             bool ok = true;
-            bool any = false;
-            for (int u = first_unit; ok && u < p.units; u += unit_step) {
-                const Unit w = unit_at<VARLEN>(p, u);
-                if (w.n_kv == 0)
+            for (int i = 0; ok; ++i) {
+                const Item w = item_at<VARLEN>(p, cta, i);
+                if (!w.ok)
+                    break;
+                const int n = w.j1 - w.j0;
+                if (n == 0)
                     continue;
-                if (!any) {
-                    ok = wait_bounded(bar(L::B_FULL + 0), 0, abort_flag, limit);   // K_0 of the first unit
-                    any = true;
-                }
+                if (iq == 0)
+                    ok = wait_bounded(bar(L::B_FULL + 0), 0, abort_flag, limit);   // first key tile
                 ok = ok && wait_bounded(bar(L::B_Q + 0), iq & 1, abort_flag, limit) &&
                      wait_bounded(bar(L::B_Q + 1), iq & 1, abort_flag, limit);
                 if (!ok)
                     break;
-                // K_0 sits in the stage before this unit's first.
+                // The item's first key tile sits in the stage before its first.
                 const int st_k0 = (g - 1) % L::NSTAGE;
                 ptx::tc_fence_after_sync();
                 issue_qk<D>(s0, dq0, dk + st_k0 * STAGE16);
                 ptx::mma_commit(bar(L::B_S + 0));
                 issue_qk<D>(s1, dq1, dk + st_k0 * STAGE16);
                 ptx::mma_commit(bar(L::B_S + 1));
-                // That stage also carried the previous unit's last V: both are done now.
+                // That stage also carried the previous item's last V: both are done now.
                 ptx::mma_commit(bar(L::B_EMPTY + st_k0));
-                if (w.n_kv == 1) {
+                if (n == 1) {
                     ptx::mma_commit(bar(L::B_QE + 0));
                     ptx::mma_commit(bar(L::B_QE + 1));
                 }
-                for (int j = 0; j < w.n_kv; ++j, ++pc) {
-                    const int st = (g + j) % L::NSTAGE;
+                for (int r = 0; r < n; ++r, ++pc) {
+                    const int st = (g + r) % L::NSTAGE;
                     const uint64_t vd = dv + st * STAGE16;
                     const uint64_t kd = dk + st * STAGE16;
-                    const bool more = j + 1 < w.n_kv;
+                    const bool more = r + 1 < n;
                     if (!(ok = wait_bounded(bar(L::B_P + 0), pc & 1, abort_flag, limit)))
                         break;
-                    if (j == 0 && iq > 0 && !(ok = wait_bounded(bar(L::B_OE + 0), (iq - 1) & 1, abort_flag, limit)))
+                    if (r == 0 && iq > 0 && !(ok = wait_bounded(bar(L::B_OE + 0), (iq - 1) & 1, abort_flag, limit)))
                         break;
                     ptx::tc_fence_after_sync();
-                    issue_pv<D>(o0, s0, vd, j > 0);
+                    issue_pv<D>(o0, s0, vd, r > 0);
                     if (more) {
                         issue_qk<D>(s0, dq0, kd);
                         ptx::mma_commit(bar(L::B_S + 0));
-                        if (j + 2 == w.n_kv)
+                        if (r + 2 == n)
                             ptx::mma_commit(bar(L::B_QE + 0));
                     } else {
                         ptx::mma_commit(bar(L::B_O + 0));
                     }
                     if (!(ok = wait_bounded(bar(L::B_P + 1), pc & 1, abort_flag, limit)))
                         break;
-                    if (j == 0 && iq > 0 && !(ok = wait_bounded(bar(L::B_OE + 1), (iq - 1) & 1, abort_flag, limit)))
+                    if (r == 0 && iq > 0 && !(ok = wait_bounded(bar(L::B_OE + 1), (iq - 1) & 1, abort_flag, limit)))
                         break;
                     ptx::tc_fence_after_sync();
-                    issue_pv<D>(o1, s1, vd, j > 0);
+                    issue_pv<D>(o1, s1, vd, r > 0);
                     if (more) {
                         issue_qk<D>(s1, dq1, kd);
                         ptx::mma_commit(bar(L::B_S + 1));
-                        if (j + 2 == w.n_kv)
+                        if (r + 2 == n)
                             ptx::mma_commit(bar(L::B_QE + 1));
                         ptx::mma_commit(bar(L::B_EMPTY + st));
                     } else {
                         ptx::mma_commit(bar(L::B_O + 1));
                     }
                 }
-                g += w.n_kv;
+                g += n;
                 ++iq;
             }
             // Retire every MMA this thread issued before TMEM is released.
@@ -525,22 +666,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // ------------------------------------------------------------ softmax warps
         const int t = warp >> 2;                 // query tile of this group
         const int wq = warp & 3;                 // TMEM lane quarter of this warp
+        const int row = wq * 32 + lane;          // query row within the tile
         const uint32_t lane_addr = tmem + (static_cast<uint32_t>(wq * 32) << 16);
         const uint32_t s_addr = lane_addr + 128 * t;
         const uint32_t o_addr = lane_addr + 256 + 128 * t;
         const float sl2 = p.scale_log2;
         const bool neg_scale = sl2 < 0.f;
-        int g = 1;      // stage of (V_0, K_1) of the current unit
+        int g = 1;      // stage of the current item's (V_j0, next K)
         int sc = 0;     // S phases consumed
-        int iq = 0;     // units with keys so far
+        int iq = 0;     // items with keys so far
         bool ok = true;
 
-        for (int u = first_unit; ok && u < p.units; u += unit_step) {
-            const Unit w = unit_at<VARLEN>(p, u);
-            const int q_row = (w.qp * 2 + t) * BM + wq * 32 + lane;
+        for (int i = 0; ok; ++i) {
+            const Item w = item_at<VARLEN>(p, cta, i);
+            if (!w.ok)
+                break;
+            const int q_row = (w.qp * 2 + t) * BM + row;
             const bool store = q_row < p.Sq;
             __nv_bfloat16 *orow = p.out + (static_cast<size_t>(w.bh) * p.Sq + (store ? q_row : 0)) * D;
-            if (w.n_kv == 0) {
+            if (w.j1 == w.j0) {
                 if (store) {
 #pragma unroll
                     for (int c = 0; c < D / 8; ++c)
@@ -553,7 +697,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             float m_used = -INFINITY;
             float l_exact = 0.f;   // sum of the fp32 weights: the log-sum-exp
             float l_resid = 0.f;   // sum over tiles of r - p for each tile's largest weight
-            for (int j = 0; j < w.n_kv; ++j, ++sc) {
+            for (int j = w.j0; j < w.j1; ++j, ++sc) {
                 if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_S + t), sc & 1, abort_flag, limit))))
                     break;
                 ptx::tc_fence_after_sync();
@@ -563,8 +707,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     ptx::tmem_ld32(s_addr + 32 * c, s[c]);
                 // The stage (V_j, next K) must have landed before P_t(j) is
                 // published; checked here, under the TMEM load latency.
-                if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + (g + j) % L::NSTAGE),
-                                                                ((g + j) / L::NSTAGE) & 1, abort_flag, limit)))) {
+                const int gj = g + (j - w.j0);
+                if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + gj % L::NSTAGE),
+                                                                (gj / L::NSTAGE) & 1, abort_flag, limit)))) {
                     ptx::tmem_wait_ld();
                     break;
                 }
@@ -599,7 +744,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 l_exact += row_probs(s, pk, sl2, neg_m);
                 ptx::tmem_st32(s_addr, pk[0]);
                 ptx::tmem_st32(s_addr + 32, pk[1]);
-                if (j > 0 && __any_sync(0xffffffffu, need)) {
+                if (j > w.j0 && __any_sync(0xffffffffu, need)) {
                     // O_t is idle here: S_t(j) was committed after PV_t(j-1), and
                     // PV_t(j) waits for the arrive below.  Done after P so that the
                     // logits' registers are free.
@@ -609,8 +754,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         ptx::tmem_ld32(o_addr + 32 * c, r);
                         ptx::tmem_wait_ld();
 #pragma unroll
-                        for (int i = 0; i < 32; ++i)
-                            r[i] = __float_as_uint(__uint_as_float(r[i]) * factor);
+                        for (int k2 = 0; k2 < 32; ++k2)
+                            r[k2] = __float_as_uint(__uint_as_float(r[k2]) * factor);
                         ptx::tmem_st32(o_addr + 32 * c, r);
                     }
                 }
@@ -627,45 +772,72 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_O + t), iq & 1, abort_flag, limit))))
                 break;
             ptx::tc_fence_after_sync();
-            const float inv_l = 1.f / (l_exact + l_resid);
-            uint32_t w16[D / 32][16];
+            if (w.part >= 0) {
+                // Part of a split tail unit: the unnormalised fp32 accumulator
+                // and this row's statistics go to the workspace; the last part
+                // to finish merges the parts of the unit.
+                const int slot = (w.tail * p.split_parts + w.part) * 2 + t;
+                float *orow_ws = p.ws_o + (static_cast<size_t>(slot) * BM + row) * D;
 #pragma unroll
-            for (int c = 0; c < D / 32; ++c) {
-                uint32_t r[32];
-                ptx::tmem_ld32(o_addr + 32 * c, r);
-                ptx::tmem_wait_ld();
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t r[32];
+                    ptx::tmem_ld32(o_addr + 32 * c, r);
+                    ptx::tmem_wait_ld();
 #pragma unroll
-                for (int i = 0; i < 16; ++i)
-                    w16[c][i] = pack_bf16x2(__uint_as_float(r[2 * i]) * inv_l, __uint_as_float(r[2 * i + 1]) * inv_l);
-            }
-            // O_t is in registers: hand the accumulator to the next unit's GEMMs
-            // before the global stores.
-            ptx::tc_fence_before_sync();
-            __syncwarp();
-            if (lane == 0)
-                ptx::mbar_arrive(bar(L::B_OE + t));
-            if (store) {
-                if (p.out_align32) {
-                    // 32-byte stores: each fills a whole sector of the row.
-#pragma unroll
-                    for (int c = 0; c < D / 32; ++c)
-#pragma unroll
-                        for (int v = 0; v < 2; ++v)
-                            ptx::st_global_v8(orow + 32 * c + 16 * v, &w16[c][8 * v]);
-                } else {
-#pragma unroll
-                    for (int c = 0; c < D / 32; ++c) {
-                        uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * c);
-#pragma unroll
-                        for (int v = 0; v < 4; ++v)
-                            dst[v] = make_uint4(w16[c][4 * v], w16[c][4 * v + 1], w16[c][4 * v + 2], w16[c][4 * v + 3]);
-                    }
+                    for (int v = 0; v < 4; ++v)
+                        ptx::st_global_v8(orow_ws + 32 * c + 8 * v, &r[8 * v]);
                 }
-                if (p.lse)
-                    p.lse[static_cast<size_t>(w.bh) * p.Sq + q_row] =
-                        (m_used + __log2f(l_exact)) * 0.69314718055994530942f;
+                reinterpret_cast<float4 *>(p.ws_stats)[slot * BM + row] = make_float4(m_used, l_exact, l_resid, 0.f);
+                ptx::tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0)
+                    ptx::mbar_arrive(bar(L::B_OE + t));
+                merge_tail_parts<D>(p, w.tail, t, row, q_row, w.bh, store, orow,
+                                    reinterpret_cast<volatile int *>(sm + L::MERGE_OFF), bar(L::B_MERGE),
+                                    bar(L::B_MERGE + 1), abort_flag);
+            } else {
+                const float inv_l = 1.f / (l_exact + l_resid);
+                uint32_t w16[D / 32][16];
+#pragma unroll
+                for (int c = 0; c < D / 32; ++c) {
+                    uint32_t r[32];
+                    ptx::tmem_ld32(o_addr + 32 * c, r);
+                    ptx::tmem_wait_ld();
+#pragma unroll
+                    for (int k2 = 0; k2 < 16; ++k2)
+                        w16[c][k2] = pack_bf16x2(__uint_as_float(r[2 * k2]) * inv_l,
+                                                 __uint_as_float(r[2 * k2 + 1]) * inv_l);
+                }
+                // O_t is in registers: hand the accumulator to the next item's
+                // GEMMs before the global stores.
+                ptx::tc_fence_before_sync();
+                __syncwarp();
+                if (lane == 0)
+                    ptx::mbar_arrive(bar(L::B_OE + t));
+                if (store) {
+                    if (p.out_align32) {
+                        // 32-byte stores: each fills a whole sector of the row.
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c)
+#pragma unroll
+                            for (int v = 0; v < 2; ++v)
+                                ptx::st_global_v8(orow + 32 * c + 16 * v, &w16[c][8 * v]);
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < D / 32; ++c) {
+                            uint4 *dst = reinterpret_cast<uint4 *>(orow + 32 * c);
+#pragma unroll
+                            for (int v = 0; v < 4; ++v)
+                                dst[v] = make_uint4(w16[c][4 * v], w16[c][4 * v + 1], w16[c][4 * v + 2],
+                                                    w16[c][4 * v + 3]);
+                        }
+                    }
+                    if (p.lse)
+                        p.lse[static_cast<size_t>(w.bh) * p.Sq + q_row] =
+                            (m_used + __log2f(l_exact)) * 0.69314718055994530942f;
+                }
             }
-            g += w.n_kv;
+            g += w.j1 - w.j0;
             ++iq;
         }
     }

@@ -3,14 +3,17 @@
 // Validation happens before any CUDA call; then, once per device, the device
 // is checked to be sm_103 and the kernels' shared-memory limits are raised;
 // then three 3-D TMA tensor maps (head dim, sequence, batch*head) are encoded
-// and one kernel is launched on the caller's stream.  Nothing is allocated.
+// and one kernel is launched on the caller's stream.  The only allocation is
+// the split-tail workspace (per device and stream, made once, kept).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <climits>
 #include <cmath>
 #include <cstdint>
+#include <map>
 #include <mutex>
+#include <utility>
 
 #include "attn_fwd_kernel.cuh"
 #include "vdx.h"
@@ -90,6 +93,36 @@ int device_ready(int *sms = nullptr)
         *sms = st.sms;
     return st.status;
 }
+
+// Workspace of the split tail, one per (device, stream): calls on one stream
+// run in order, so they can share it; calls on different streams never do.
+// Allocated on the first call that needs it, grown when a later call needs
+// more (cudaFree waits for work still using the old one), kept until exit.
+struct Workspace {
+    void *ptr = nullptr;
+    size_t bytes = 0;
+};
+std::mutex g_ws_mutex;
+std::map<std::pair<int, cudaStream_t>, Workspace> g_ws;
+
+int workspace(int dev, cudaStream_t stream, size_t bytes, void **out)
+{
+    std::lock_guard<std::mutex> lock(g_ws_mutex);
+    Workspace &w = g_ws[{dev, stream}];
+    if (w.bytes < bytes) {
+        if (w.ptr && cudaFree(w.ptr) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        w.ptr = nullptr;
+        w.bytes = 0;
+        if (cudaMalloc(&w.ptr, bytes) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        w.bytes = bytes;
+    }
+    *out = w.ptr;
+    return VDX_OK;
+}
+
+size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 // [B*H, rows, D] bf16 tensor as a 3-D TMA map with 64 x 128 x 1 boxes, 128-B swizzle.
 int make_map(CUtensorMap *map, const void *base, long long rows, long long bh, int D)
@@ -177,9 +210,39 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     // Persistent grid: one CTA per multiprocessor (one fits per SM), each
     // taking units blockIdx.x, blockIdx.x + grid, ... so that the CTAs
     // running at any moment work on neighbouring units of the same heads.
-    const dim3 grid(static_cast<unsigned>(p.units < sms ? p.units : sms));
+    const int G = p.units < sms ? p.units : sms;
+    const dim3 grid(static_cast<unsigned>(G));
     const dim3 block(vdx::NUM_THREADS);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
+
+    // Short last round: when at most half the CTAs would get a unit in it,
+    // cut each of those units along the keys into parts, one per CTA, and
+    // merge the parts (dense problems; varlen units vary in length).
+    const int n_kv = (Skv + vdx::BN - 1) / vdx::BN;
+    const int full_rounds = p.units / G;
+    const int tail = p.units - full_rounds * G;
+    int parts = (!varlen && full_rounds >= 1 && tail > 0) ? G / tail : 0;
+    if (parts > n_kv)
+        parts = n_kv;
+    if (parts >= 2) {
+        const size_t o_bytes = round_up(static_cast<size_t>(tail) * parts * 2 * vdx::BM * D * 4, 256);
+        const size_t st_bytes = round_up(static_cast<size_t>(tail) * parts * 2 * vdx::BM * 16, 256);
+        const size_t cnt_bytes = round_up(static_cast<size_t>(tail) * 4, 256);
+        int dev = 0;
+        void *ws = nullptr;
+        if (cudaGetDevice(&dev) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        if ((st = workspace(dev, s, o_bytes + st_bytes + cnt_bytes, &ws)) != VDX_OK)
+            return st;
+        p.split_parts = parts;
+        p.full_rounds = full_rounds;
+        p.tail_units = tail;
+        p.ws_o = static_cast<float *>(ws);
+        p.ws_stats = reinterpret_cast<float *>(static_cast<char *>(ws) + o_bytes);
+        p.ws_count = reinterpret_cast<int *>(static_cast<char *>(ws) + o_bytes + st_bytes);
+        if (cudaMemsetAsync(p.ws_count, 0, static_cast<size_t>(tail) * 4, s) != cudaSuccess)
+            return VDX_ERR_CUDA;
+    }
     if (D == 128) {
         if (varlen)
             vdx::attn_fwd_kernel<128, true><<<grid, block, vdx::Layout<128>::ALLOC, s>>>(mq, mk, mv, p);

@@ -148,3 +148,30 @@ def test_varlen_many_units_mixed_lengths():
     the units every CTA walks."""
     lens = np.array([0, 300, 1, 129, 0, 256, 64, 255], np.int32)
     check_case(8, 20, 257, 300, 128, 128 ** -0.5, seed=501, kv_lens=lens)
+
+
+# A short last round: with 152 SMs these leave 2 and 8 units for the last
+# round, which the library splits along the keys into parts on idle CTAs and
+# merges through its workspace (16 parts of one key tile, 8 parts with a
+# ragged last key tile).
+SPLIT_TAIL = [
+    # B, H, Sq, Skv, D
+    (1, 154, 256, 2000, 128),
+    (2, 80, 100, 1000, 64),
+    (1, 153, 200, 300, 128),
+]
+
+
+@pytest.mark.parametrize("B,H,Sq,Skv,D", SPLIT_TAIL)
+def test_split_tail(B, H, Sq, Skv, D):
+    check_case(B, H, Sq, Skv, D, 1 / math.sqrt(D), seed=600 + H + Skv, gain=1.6)
+
+
+def test_split_tail_deterministic_and_lse_optional():
+    from paper_2609_18077_gb300 import workloads
+    q, k, v = workloads.random_qkv(1, 154, 256, 2000, 128, seed=7, logit_gain=1.6)
+    o1, l1 = run_gpu(q, k, v, 128 ** -0.5)
+    o2, l2 = run_gpu(q, k, v, 128 ** -0.5)
+    assert torch.equal(o1, o2) and torch.equal(l1, l2)
+    o3, l3 = run_gpu(q, k, v, 128 ** -0.5, with_lse=False)
+    assert l3 is None and torch.equal(o3, o1)
