@@ -81,6 +81,33 @@ int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, 
                         int B, int H, int Sq, int Skv_max, int D, const int *kv_lens,
                         float scale, void *stream);
 
+/*
+ * vdx_attn_fwd without any device allocation (the paper has no counterpart;
+ * this is a library service).  Same arguments, results and errors as
+ * vdx_attn_fwd, for callers that must not allocate device memory: code that
+ * runs where cudaMalloc is not allowed or would stall the device (a stream
+ * being captured into a graph, a serving loop whose memory is planned up
+ * front, a process whose device memory belongs to another allocator).
+ *
+ * Instead of the library's per-stream workspace, the split-tail scratch lives
+ * in a fixed 24 MiB array of device memory inside the library image, which
+ * every GPU that loads the library holds until the process exits.  A call
+ * whose scratch need exceeds 24 MiB returns VDX_ERR_UNSUPPORTED and launches
+ * nothing (with at most one part per multiprocessor the need stays near
+ * 21 MB at D = 128 on a 152-SM GB300).
+ *
+ * The first call on a device also looks up that array's device address
+ * (once per device, the device being current); make that first call before
+ * any stream capture.  Every call on a device shares the one array and it
+ * keeps the previous call's contents: each call clears its counters itself,
+ * on its stream, before the kernel.  Calls whose work overlaps on the GPU
+ * (different streams, or threads without ordering) race on the array, so
+ * order them.  No cudaMalloc, cudaFree or allocating library routine is
+ * called.
+ */
+int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out, float *lse,
+                         int B, int H, int Sq, int Skv, int D, float scale, void *stream);
+
 /* Human-readable name of a vdx_status (static storage; never NULL). */
 const char *vdx_status_string(int status);
 

@@ -31,6 +31,7 @@ _I = ctypes.c_int
 SIGNATURES = {
     "vdx_attn_fwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, ctypes.c_float, _P]),
     "vdx_attn_fwd_varlen": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, ctypes.c_float, _P]),
+    "vdx_attn_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, ctypes.c_float, _P]),
     "vdx_status_string": (ctypes.c_char_p, [_I]),
     "vdx_check_device_error": (_I, [_P]),
     "vdx_selftest_wait_timeout": (_I, [_I, _P]),

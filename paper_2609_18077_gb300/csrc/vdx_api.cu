@@ -146,8 +146,11 @@ bool overlaps(const void *a, size_t na, const void *b, size_t nb)
     return x < y + nb && y < x + na;
 }
 
+// fixed_scratch / fixed_bytes: when set, the split-tail workspace is taken
+// from that fixed device region instead of the library's allocation.
 int attn_launch(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
-                int D, const int *kv_lens, bool varlen, float scale, void *stream)
+                int D, const int *kv_lens, bool varlen, float scale, void *stream, void *fixed_scratch = nullptr,
+                size_t fixed_bytes = 0)
 {
     // ---- validation (no CUDA calls)
     if (!q || !k || !v || !out || (varlen && !kv_lens))
@@ -232,8 +235,13 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         void *ws = nullptr;
         if (cudaGetDevice(&dev) != cudaSuccess)
             return VDX_ERR_CUDA;
-        if ((st = workspace(dev, s, o_bytes + st_bytes + cnt_bytes, &ws)) != VDX_OK)
+        if (fixed_scratch) {
+            if (o_bytes + st_bytes + cnt_bytes > fixed_bytes)
+                return VDX_ERR_UNSUPPORTED;
+            ws = fixed_scratch;
+        } else if ((st = workspace(dev, s, o_bytes + st_bytes + cnt_bytes, &ws)) != VDX_OK) {
             return st;
+        }
         p.split_parts = parts;
         p.full_rounds = full_rounds;
         p.tail_units = tail;
@@ -260,9 +268,67 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     return e == cudaSuccess ? VDX_OK : VDX_ERR_CUDA;
 }
 
+// ---------------------------------------------------------------- no-allocation variant
+// Scratch for vdx_attn_fwd_noalloc: a fixed array in device memory, part of
+// the library image, so every GPU that loads the library holds these 24 MiB
+// until the process exits.  24 MiB covers the split-tail workspace of any
+// call on a GPU with up to 152 multiprocessors (at most one part per
+// multiprocessor: 152 x 2 x 128 x (4 x 128 + 16) bytes ~ 20.6 MB at D = 128).
+constexpr size_t kNoAllocScratchBytes = size_t(24) << 20;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+// In host code `g_noalloc_scratch` names a host-side stand-in, not the device
+// array, so its device address is looked up once per device (that device
+// current) and passed to the kernel.
+struct NoAllocState {
+    std::once_flag once;
+    int status = VDX_OK;
+    void *ptr = nullptr;
+};
+NoAllocState g_noalloc[kMaxDevices];
+
+int noalloc_scratch(void **ptr)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices)
+        return VDX_ERR_UNSUPPORTED;
+    NoAllocState &st = g_noalloc[dev];
+    std::call_once(st.once, [&] {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) {
+            st.status = VDX_ERR_CUDA;
+            return;
+        }
+        st.ptr = p;
+    });
+    *ptr = st.ptr;
+    return st.status;
+}
+
 }  // namespace
 
 extern "C" {
+
+int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,
+                         int Skv, int D, float scale, void *stream)
+{
+    // Argument checks first, exactly as vdx_attn_fwd does them, so a bad call
+    // touches no CUDA state; then the fixed scratch's device address.
+    if (!q || !k || !v || !out || B < 0 || H < 0 || Sq < 0 || Skv < 0 || (D != 64 && D != 128) ||
+        !std::isfinite(scale))
+        return VDX_ERR_INVALID_ARG;
+    if (static_cast<long long>(B) * H == 0 || Sq == 0)
+        return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, nullptr, false, scale, stream);
+    void *scratch = nullptr;
+    const int st = noalloc_scratch(&scratch);
+    if (st != VDX_OK)
+        return st;
+    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, nullptr, false, scale, stream, scratch,
+                       kNoAllocScratchBytes);
+}
+
 
 int vdx_attn_fwd(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
                  int D, float scale, void *stream)
