@@ -93,19 +93,21 @@ struct AttnParams {
     uint64_t wait_limit_ns;
 };
 
-template <int D>
+// Shared-memory plan.  QBUF Q-tile pairs (2 = the next item's Q tiles load
+// while the current item runs) and NSTAGE K/V stages of (V_j, next K).
+template <int D, int QBUF, int NSTAGE_>
 struct Layout {
     static_assert(D == 64 || D == 128, "head dim");
     static constexpr int TILE_BYTES = BM * D * 2;           // one Q, K or V tile
     static constexpr int HALF_BYTES = BM * 128;              // one 64-column swizzle block
-    static constexpr int NSTAGE = D == 128 ? 2 : 4;          // K/V ring: stage = (V_j, K_{j+1})
-    static constexpr int Q_OFF = 0;
-    static constexpr int KV_OFF = 2 * TILE_BYTES;            // stage s: V at 2s, K at 2s+1 (tiles)
+    static constexpr int NSTAGE = NSTAGE_;                   // K/V ring: stage = (V_j, next K)
+    static constexpr int Q_OFF = 0;                          // Q buffer b, tile t at (2b + t) tiles
+    static constexpr int KV_OFF = 2 * QBUF * TILE_BYTES;     // stage s: V at 2s, K at 2s+1 (tiles)
     static constexpr int BAR_OFF = KV_OFF + 2 * NSTAGE * TILE_BYTES;
     // barrier indices
-    static constexpr int B_Q = 0;                            // [2] Q tile t landed
-    static constexpr int B_QE = 2;                           // [2] Q tile t free (last QK^T of a unit ran)
-    static constexpr int B_FULL = 4;                         // [NSTAGE] stage landed
+    static constexpr int B_Q = 0;                            // [2 QBUF] Q tile (buffer b, tile t) landed
+    static constexpr int B_QE = 2 * QBUF;                    // [2 QBUF] that Q tile free (its last QK^T ran)
+    static constexpr int B_FULL = 4 * QBUF;                  // [NSTAGE] stage landed
     static constexpr int B_EMPTY = B_FULL + NSTAGE;          // [NSTAGE] stage consumed
     static constexpr int B_S = B_EMPTY + NSTAGE;             // [2] S_t ready
     static constexpr int B_P = B_S + 2;                      // [2] P_t written, O_t rescaled
@@ -211,7 +213,7 @@ __device__ __forceinline__ void issue_qk(uint32_t s_tmem, uint64_t q_desc, uint6
     constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, BN, 0);
 #pragma unroll
     for (int kk = 0; kk < D / 16; ++kk) {
-        const uint32_t off = ((kk >> 2) * Layout<D>::HALF_BYTES + (kk & 3) * 32) >> 4;
+        const uint32_t off = ((kk >> 2) * (BM * 128) + (kk & 3) * 32) >> 4;
         ptx::mma_ss(s_tmem, q_desc + off, k_desc + off, idesc, kk > 0);
     }
 }
@@ -410,12 +412,12 @@ __device__ __forceinline__ Item item_at(const AttnParams &p, int cta, int i)
     return w;
 }
 
-template <int D, bool VARLEN>
+template <int D, bool VARLEN, int QBUF, int NSTAGE>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
                     const __grid_constant__ CUtensorMap tmap_v, const AttnParams p)
 {
-    using L = Layout<D>;
+    using L = Layout<D, QBUF, NSTAGE>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const uint32_t sbase = ptx::smem_u32(sm);
@@ -427,9 +429,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     const int cta = blockIdx.x;
 
     if (threadIdx.x == 0) {
+        for (int b = 0; b < 2 * QBUF; ++b) {
+            ptx::mbar_init(bar(L::B_Q + b), 1);
+            ptx::mbar_init(bar(L::B_QE + b), 1);
+        }
         for (int t = 0; t < 2; ++t) {
-            ptx::mbar_init(bar(L::B_Q + t), 1);
-            ptx::mbar_init(bar(L::B_QE + t), 1);
             ptx::mbar_init(bar(L::B_S + t), 1);
             ptx::mbar_init(bar(L::B_P + t), 4);    // one arrive per softmax warp
             ptx::mbar_init(bar(L::B_O + t), 1);
@@ -547,19 +551,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         for (int iq = 0; ok && i >= 0; ++iq) {
             const Item w = item_at<VARLEN>(p, cta, i);
             const int ni = next_with_keys(i);
-            if (iq > 0) {
-                // Q tiles of the previous item are free once its last QK^T ran.
-                ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_QE + 0), (iq - 1) & 1, abort_flag, limit) &&
-                                                 wait_bounded(bar(L::B_QE + 1), (iq - 1) & 1, abort_flag, limit));
+            const int qb = iq % QBUF;
+            if (iq >= QBUF) {
+                // Q buffer qb is free once its previous item's last QK^T ran.
+                const int ph = ((iq / QBUF) - 1) & 1;
+                ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_QE + 2 * qb), ph, abort_flag, limit) &&
+                                                 wait_bounded(bar(L::B_QE + 2 * qb + 1), ph, abort_flag, limit));
                 if (!ok)
                     break;
             }
             if (lane == 0) {
                 for (int t = 0; t < 2; ++t) {
-                    ptx::mbar_arrive_expect_tx(bar(L::B_Q + t), L::TILE_BYTES);
+                    ptx::mbar_arrive_expect_tx(bar(L::B_Q + 2 * qb + t), L::TILE_BYTES);
                     for (int h = 0; h < D / 64; ++h)
-                        ptx::tma_load_3d(sbase + L::Q_OFF + t * L::TILE_BYTES + h * L::HALF_BYTES, &tmap_q,
-                                         bar(L::B_Q + t), h * 64, (w.qp * 2 + t) * BM, w.bh);
+                        ptx::tma_load_3d(sbase + L::Q_OFF + (2 * qb + t) * L::TILE_BYTES + h * L::HALF_BYTES,
+                                         &tmap_q, bar(L::B_Q + 2 * qb + t), h * 64, (w.qp * 2 + t) * BM, w.bh);
                 }
             }
             Item nw;
@@ -577,8 +583,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
     } else if (warp == MMA_WARP) {
         // ------------------------------------------------------------ tcgen05 issuer
         if (lane == 0) {
-            const uint64_t dq0 = ptx::smem_desc_sw128(sbase + L::Q_OFF, 16, 1024);
-            const uint64_t dq1 = ptx::smem_desc_sw128(sbase + L::Q_OFF + L::TILE_BYTES, 16, 1024);
+            const uint64_t dq_base = ptx::smem_desc_sw128(sbase + L::Q_OFF, 16, 1024);
+            constexpr uint32_t TILE16 = L::TILE_BYTES >> 4;
             const uint64_t dk = ptx::smem_desc_sw128(sbase + L::KV_OFF + L::TILE_BYTES, 16, 1024);
             const uint64_t dv = ptx::smem_desc_sw128(sbase + L::KV_OFF, L::HALF_BYTES, 1024);
             constexpr uint32_t STAGE16 = (2 * L::TILE_BYTES) >> 4;
@@ -596,10 +602,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     continue;
                 if (iq == 0)
                     ok = wait_bounded(bar(L::B_FULL + 0), 0, abort_flag, limit);   // first key tile
-                ok = ok && wait_bounded(bar(L::B_Q + 0), iq & 1, abort_flag, limit) &&
-                     wait_bounded(bar(L::B_Q + 1), iq & 1, abort_flag, limit);
+                const int qb = iq % QBUF;
+                const int qph = (iq / QBUF) & 1;
+                ok = ok && wait_bounded(bar(L::B_Q + 2 * qb), qph, abort_flag, limit) &&
+                     wait_bounded(bar(L::B_Q + 2 * qb + 1), qph, abort_flag, limit);
                 if (!ok)
                     break;
+                const uint64_t dq0 = dq_base + (2 * qb) * TILE16;
+                const uint64_t dq1 = dq_base + (2 * qb + 1) * TILE16;
                 // The item's first key tile sits in the stage before its first.
                 const int st_k0 = (g - 1) % L::NSTAGE;
                 ptx::tc_fence_after_sync();
@@ -610,8 +620,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 // That stage also carried the previous item's last V: both are done now.
                 ptx::mma_commit(bar(L::B_EMPTY + st_k0));
                 if (n == 1) {
-                    ptx::mma_commit(bar(L::B_QE + 0));
-                    ptx::mma_commit(bar(L::B_QE + 1));
+                    ptx::mma_commit(bar(L::B_QE + 2 * qb));
+                    ptx::mma_commit(bar(L::B_QE + 2 * qb + 1));
                 }
                 for (int r = 0; r < n; ++r, ++pc) {
                     const int st = (g + r) % L::NSTAGE;
@@ -628,7 +638,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         issue_qk<D>(s0, dq0, kd);
                         ptx::mma_commit(bar(L::B_S + 0));
                         if (r + 2 == n)
-                            ptx::mma_commit(bar(L::B_QE + 0));
+                            ptx::mma_commit(bar(L::B_QE + 2 * qb));
                     } else {
                         ptx::mma_commit(bar(L::B_O + 0));
                     }
@@ -642,7 +652,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         issue_qk<D>(s1, dq1, kd);
                         ptx::mma_commit(bar(L::B_S + 1));
                         if (r + 2 == n)
-                            ptx::mma_commit(bar(L::B_QE + 1));
+                            ptx::mma_commit(bar(L::B_QE + 2 * qb + 1));
                         ptx::mma_commit(bar(L::B_EMPTY + st));
                     } else {
                         ptx::mma_commit(bar(L::B_O + 1));

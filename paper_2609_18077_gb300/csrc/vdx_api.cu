@@ -50,11 +50,37 @@ struct DeviceState {
 };
 DeviceState g_devices[kMaxDevices];
 
-template <int D, bool VARLEN>
+// Kernel configurations: (Q buffers, K/V stages) per head dim.  D = 128 fits
+// one Q buffer and two K/V stages (a second Q buffer would leave one stage,
+// which serialises the K/V loads and measured slower even on the two-tile
+// text cross-attention); D = 64 fits two Q buffers (the next item's Q loads a
+// whole item ahead) and four stages.
+
+template <int D, bool VARLEN, int QBUF, int NSTAGE>
 cudaError_t raise_smem_limit()
 {
-    return cudaFuncSetAttribute(vdx::attn_fwd_kernel<D, VARLEN>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                vdx::Layout<D>::ALLOC);
+    return cudaFuncSetAttribute(vdx::attn_fwd_kernel<D, VARLEN, QBUF, NSTAGE>,
+                                cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                vdx::Layout<D, QBUF, NSTAGE>::ALLOC);
+}
+
+cudaError_t raise_all_smem_limits()
+{
+    cudaError_t e = cudaSuccess;
+    for (cudaError_t r : {raise_smem_limit<128, false, 1, 2>(), raise_smem_limit<128, true, 1, 2>(),
+                          raise_smem_limit<64, false, 2, 4>(), raise_smem_limit<64, true, 2, 4>()})
+        if (r != cudaSuccess)
+            e = r;
+    return e;
+}
+
+template <int D, bool VARLEN, int QBUF, int NSTAGE>
+cudaError_t launch(dim3 grid, const CUtensorMap &mq, const CUtensorMap &mk, const CUtensorMap &mv,
+                   const vdx::AttnParams &p, cudaStream_t s)
+{
+    vdx::attn_fwd_kernel<D, VARLEN, QBUF, NSTAGE>
+        <<<grid, vdx::NUM_THREADS, vdx::Layout<D, QBUF, NSTAGE>::ALLOC, s>>>(mq, mk, mv, p);
+    return cudaGetLastError();
 }
 
 // One-time per-device check and kernel attribute set-up (current device).
@@ -82,8 +108,7 @@ int device_ready(int *sms = nullptr)
             st.status = VDX_ERR_CUDA;
             return;
         }
-        if (raise_smem_limit<64, false>() != cudaSuccess || raise_smem_limit<64, true>() != cudaSuccess ||
-            raise_smem_limit<128, false>() != cudaSuccess || raise_smem_limit<128, true>() != cudaSuccess) {
+        if (raise_all_smem_limits() != cudaSuccess) {
             st.status = VDX_ERR_CUDA;
             return;
         }
@@ -215,7 +240,6 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     // running at any moment work on neighbouring units of the same heads.
     const int G = p.units < sms ? p.units : sms;
     const dim3 grid(static_cast<unsigned>(G));
-    const dim3 block(vdx::NUM_THREADS);
     cudaStream_t s = static_cast<cudaStream_t>(stream);
 
     // Short last round: when at most half the CTAs would get a unit in it,
@@ -251,18 +275,12 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         if (cudaMemsetAsync(p.ws_count, 0, static_cast<size_t>(tail) * 4, s) != cudaSuccess)
             return VDX_ERR_CUDA;
     }
+    cudaError_t e;
     if (D == 128) {
-        if (varlen)
-            vdx::attn_fwd_kernel<128, true><<<grid, block, vdx::Layout<128>::ALLOC, s>>>(mq, mk, mv, p);
-        else
-            vdx::attn_fwd_kernel<128, false><<<grid, block, vdx::Layout<128>::ALLOC, s>>>(mq, mk, mv, p);
+        e = varlen ? launch<128, true, 1, 2>(grid, mq, mk, mv, p, s) : launch<128, false, 1, 2>(grid, mq, mk, mv, p, s);
     } else {
-        if (varlen)
-            vdx::attn_fwd_kernel<64, true><<<grid, block, vdx::Layout<64>::ALLOC, s>>>(mq, mk, mv, p);
-        else
-            vdx::attn_fwd_kernel<64, false><<<grid, block, vdx::Layout<64>::ALLOC, s>>>(mq, mk, mv, p);
+        e = varlen ? launch<64, true, 2, 4>(grid, mq, mk, mv, p, s) : launch<64, false, 2, 4>(grid, mq, mk, mv, p, s);
     }
-    const cudaError_t e = cudaGetLastError();
     if (e == cudaErrorNoKernelImageForDevice)
         return VDX_ERR_DEVICE;
     return e == cudaSuccess ? VDX_OK : VDX_ERR_CUDA;
