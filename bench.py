@@ -253,7 +253,8 @@ def run_ours(args):
                      "peak_kind": f"{peak_kind} bf16 dense burst",
                      "frac_of_sustained": round(per_launch_tflops / float(peaks["bf16_tflops_sustained"]), 4),
                      "traffic": traffic,
-                     "kernel": "vdx::attn_fwd_kernel<%d,%s>" % (wl.D, "true" if lens is not None else "false")},
+                     "kernel": "vdx::attn_fwd_kernel<%d,%s,%s>" % (wl.D, "true" if lens is not None else "false",
+                                                                      "1,2" if wl.D == 128 else "2,4")},
         "cpu_baseline": cpu,
     }
     print(json.dumps(line), flush=True)
