@@ -8,7 +8,8 @@ and this package imports nothing from it.
 What the oracle computes is the plain softmax-attention definition (vidax
 paper, Sec. 2 "3D RoPE, 3D VAEs, and flash attention": flash attention is
 an exact re-ordering of it), with padded text keys excluded per sample
-(appendix Table 4, segment-id masking of invalid key blocks).  See the
+(appendix Table 4, segment-id masking of invalid key blocks), either as a
+valid key count per sample or as segment ids per token.  See the
 header of ``oracle.c`` for the formulas.
 
 Inputs are bf16 bit patterns as ``numpy.uint16`` arrays ``[B, H, S, D]``;
@@ -49,6 +50,12 @@ class Oracle:
             ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
             ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
             ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
+        lib.oracle_attn_fwd_seg.restype = ctypes.c_int
+        lib.oracle_attn_fwd_seg.argtypes = [
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+            ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
         lib.oracle_set_threads.restype = ctypes.c_int
         lib.oracle_set_threads.argtypes = [ctypes.c_int]
         self._lib = lib
@@ -57,12 +64,14 @@ class Oracle:
         """Set the OpenMP thread count (n <= 0 keeps it); returns the count in use."""
         return int(self._lib.oracle_set_threads(int(n)))
 
-    def attn_fwd(self, q, k, v, scale, kv_lens=None, rows=None, probs=False):
+    def attn_fwd(self, q, k, v, scale, kv_lens=None, rows=None, probs=False, q_seg=None, kv_seg=None):
         """Attention forward in fp64.
 
         q: uint16 [B,H,Sq,D]; k, v: uint16 [B,H,Skv,D] (bf16 bits).
         kv_lens: None or int [B] (valid keys per sample, clamped to [0, Skv]).
         rows: None (all query rows) or int [B*H, n] query indices per (b, h).
+        q_seg, kv_seg: None, or int [B,Sq] and int [B,Skv] segment ids (given
+        together, without kv_lens): a query attends the keys of its segment.
         Returns (o [B,H,n,D] f64, lse [B,H,n] f64[, probs [B,H,n,Skv] f64]).
         """
         q = _bits(q)
@@ -85,14 +94,28 @@ class Oracle:
             if rows_arr.ndim != 2 or rows_arr.shape[0] != B * H:
                 raise ValueError("rows must have shape [B*H, n]")
             n = rows_arr.shape[1]
+        if (q_seg is None) != (kv_seg is None):
+            raise ValueError("q_seg and kv_seg go together")
+        if q_seg is not None:
+            if lens is not None:
+                raise ValueError("segment ids and kv_lens are exclusive")
+            qs = np.ascontiguousarray(np.asarray(q_seg, dtype=np.int32))
+            ks = np.ascontiguousarray(np.asarray(kv_seg, dtype=np.int32))
+            if qs.shape != (B, Sq) or ks.shape != (B, Skv):
+                raise ValueError("q_seg must be [B,Sq] and kv_seg [B,Skv]")
         o = np.empty((B, H, n, D), dtype=np.float64)
         lse = np.empty((B, H, n), dtype=np.float64)
         pr = np.empty((B, H, n, Skv), dtype=np.float64) if probs else None
-        rc = self._lib.oracle_attn_fwd(
-            _ptr(q), _ptr(k), _ptr(v), B, H, Sq, Skv, D, float(scale),
-            _ptr(lens), _ptr(rows_arr), n, _ptr(o), _ptr(lse), _ptr(pr))
+        if q_seg is None:
+            rc = self._lib.oracle_attn_fwd(
+                _ptr(q), _ptr(k), _ptr(v), B, H, Sq, Skv, D, float(scale),
+                _ptr(lens), _ptr(rows_arr), n, _ptr(o), _ptr(lse), _ptr(pr))
+        else:
+            rc = self._lib.oracle_attn_fwd_seg(
+                _ptr(q), _ptr(k), _ptr(v), B, H, Sq, Skv, D, float(scale),
+                _ptr(qs), _ptr(ks), _ptr(rows_arr), n, _ptr(o), _ptr(lse), _ptr(pr))
         if rc != 0:
-            raise RuntimeError("oracle_attn_fwd rejected its arguments")
+            raise RuntimeError("oracle attention rejected its arguments")
         return (o, lse, pr) if probs else (o, lse)
 
 
@@ -120,6 +143,7 @@ def default() -> Oracle:
     return _default
 
 
-def attn_fwd(q, k, v, scale, kv_lens=None, rows=None, probs=False):
+def attn_fwd(q, k, v, scale, kv_lens=None, rows=None, probs=False, q_seg=None, kv_seg=None):
     """Module-level shortcut for ``default().attn_fwd``."""
-    return default().attn_fwd(q, k, v, scale, kv_lens=kv_lens, rows=rows, probs=probs)
+    return default().attn_fwd(q, k, v, scale, kv_lens=kv_lens, rows=rows, probs=probs, q_seg=q_seg,
+                              kv_seg=kv_seg)

@@ -26,6 +26,13 @@
  * per-batch valid key count L_b = clamp(kv_lens[b], 0, Skv); keys j >= L_b are
  * never read.  L_b = 0 gives o = 0 and lse = -inf.
  *
+ * Joint text-video attention (oracle_attn_fwd_seg) generalises the valid
+ * count to segment ids, the form the same appendix entry names for
+ * HunyuanVideo-1.5's joint attention over video and padded text tokens: query
+ * i of sample b attends exactly the keys j with kv_seg[b,j] == q_seg[b,i], and
+ * the definition above runs over that key set in ascending key order.  A query
+ * whose segment owns no key gets o = 0 and lse = -inf.
+ *
  * Inputs are bf16 bit patterns (uint16), decoded exactly to fp64.  All
  * arithmetic is fp64.  Layout: q [B,H,Sq,D], k and v [B,H,Skv,D], contiguous.
  * Parallelism: one OpenMP loop over (b, h, query row); each row is computed
@@ -49,12 +56,14 @@ static double bf16_to_f64(uint16_t bits)
 }
 
 /*
- * Attention for one query row against the first L keys of one (b, h).
- * q: D values; k, v: [L or more, D]; s: scratch of L doubles.
- * Writes o[D], *lse and, if probs != NULL, probs[j] = softmax weight of key j.
+ * Attention for one query row against L keys of one (b, h): keys 0 .. L-1,
+ * or, when idx != NULL, keys idx[0], ..., idx[L-1].
+ * q: D values; k, v: [Skv, D]; s: scratch of L doubles.
+ * Writes o[D], *lse and, if probs != NULL, probs[r] = softmax weight of the
+ * r-th attended key.
  */
 static void attend_row(const uint16_t *q, const uint16_t *k, const uint16_t *v,
-                       int L, int D, double scale, double *s,
+                       const int *idx, int L, int D, double scale, double *s,
                        double *o, double *lse, double *probs)
 {
     if (L <= 0) {
@@ -65,9 +74,10 @@ static void attend_row(const uint16_t *q, const uint16_t *k, const uint16_t *v,
     }
     /* logits */
     for (int j = 0; j < L; ++j) {
+        const size_t kj = (size_t)(idx ? idx[j] : j);
         double dot = 0.0;
         for (int d = 0; d < D; ++d)
-            dot += bf16_to_f64(q[d]) * bf16_to_f64(k[(size_t)j * D + d]);
+            dot += bf16_to_f64(q[d]) * bf16_to_f64(k[kj * D + d]);
         s[j] = scale * dot;
     }
     /* softmax normaliser */
@@ -82,11 +92,12 @@ static void attend_row(const uint16_t *q, const uint16_t *k, const uint16_t *v,
     for (int d = 0; d < D; ++d)
         o[d] = 0.0;
     for (int j = 0; j < L; ++j) {
+        const size_t vj = (size_t)(idx ? idx[j] : j);
         double p = exp(s[j] - m) / l;
         if (probs)
             probs[j] = p;
         for (int d = 0; d < D; ++d)
-            o[d] += p * bf16_to_f64(v[(size_t)j * D + d]);
+            o[d] += p * bf16_to_f64(v[vj * D + d]);
     }
     *lse = m + log(l);
 }
@@ -155,9 +166,83 @@ int oracle_attn_fwd(const uint16_t *q, const uint16_t *k, const uint16_t *v,
             if (pr)
                 for (int j = 0; j < Skv; ++j)
                     pr[j] = 0.0;
-            attend_row(qi, kb, vb, L, D, scale, s, o + (size_t)t * D, lse + t, pr);
+            attend_row(qi, kb, vb, NULL, L, D, scale, s, o + (size_t)t * D, lse + t, pr);
         }
         free(s);
+    }
+    return failed ? -1 : 0;
+}
+
+/*
+ * Joint attention with segment ids: query i of sample b attends the keys j
+ * with kv_seg[b*Skv + j] == q_seg[b*Sq + i] (see the header).
+ *
+ *   q_seg: int32 [B, Sq]; kv_seg: int32 [B, Skv] (shared by the heads).
+ *   rows, o, lse: as for oracle_attn_fwd.
+ *   probs (optional, tiny shapes only): [B*H, nrows or Sq, Skv], zero for
+ *   keys outside the row's segment.
+ *
+ * Returns 0, or -1 on a bad argument or a failed allocation.
+ */
+int oracle_attn_fwd_seg(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                        int B, int H, int Sq, int Skv, int D, double scale,
+                        const int32_t *q_seg, const int32_t *kv_seg,
+                        const int32_t *rows, int nrows,
+                        double *o, double *lse, double *probs)
+{
+    if (!q || !k || !v || !o || !lse || !q_seg || !kv_seg || B < 0 || H < 0 || Sq < 0 || Skv < 0 || D <= 0)
+        return -1;
+    const int nr = rows ? nrows : Sq;
+    if (nr < 0)
+        return -1;
+    const long total = (long)B * H * nr;
+    const size_t cap = (size_t)(Skv > 0 ? Skv : 1);
+    int failed = 0;
+
+#pragma omp parallel
+    {
+        double *s = (double *)malloc(sizeof(double) * cap);
+        double *ps = (double *)malloc(sizeof(double) * cap);
+        int *idx = (int *)malloc(sizeof(int) * cap);
+        if (!s || !ps || !idx) {
+#pragma omp atomic write
+            failed = 1;
+        }
+#pragma omp for schedule(dynamic, 4)
+        for (long t = 0; t < total; ++t) {
+            if (!s || !ps || !idx)
+                continue;
+            const long bh = t / nr;
+            const int r = (int)(t % nr);
+            const int b = (int)(bh / H);
+            const int i = rows ? rows[bh * nrows + r] : r;
+            if (i < 0 || i >= Sq) {
+#pragma omp atomic write
+                failed = 1;
+                continue;
+            }
+            /* the keys of this query's segment, in ascending order */
+            const int32_t seg = q_seg[(size_t)b * Sq + i];
+            const int32_t *kseg = kv_seg + (size_t)b * Skv;
+            int n = 0;
+            for (int j = 0; j < Skv; ++j)
+                if (kseg[j] == seg)
+                    idx[n++] = j;
+            const uint16_t *qi = q + ((size_t)bh * Sq + i) * D;
+            const uint16_t *kb = k + (size_t)bh * Skv * D;
+            const uint16_t *vb = v + (size_t)bh * Skv * D;
+            attend_row(qi, kb, vb, idx, n, D, scale, s, o + (size_t)t * D, lse + t, probs ? ps : NULL);
+            if (probs) {
+                double *pr = probs + (size_t)t * Skv;
+                for (int j = 0; j < Skv; ++j)
+                    pr[j] = 0.0;
+                for (int e = 0; e < n; ++e)
+                    pr[idx[e]] = ps[e];
+            }
+        }
+        free(s);
+        free(ps);
+        free(idx);
     }
     return failed ? -1 : 0;
 }

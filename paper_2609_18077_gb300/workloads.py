@@ -23,8 +23,15 @@ Recipe (every draw is seeded; no dataset is read):
   * text lengths: one integer per sample, uniform on the inclusive range
     [lo, hi]; K/V rows past a sample's length are padding and may be filled
     with NaN to prove they are never read;
-  * row subsets for large configs: per (b, h), n distinct query rows.
-Independent streams (lengths, outliers, row subsets) come from
+  * row subsets for large configs: per (b, h), n distinct query rows;
+  * joint text-video attention (appendix Table 4, HunyuanVideo-1.5's joint
+    attention over video and padded text, masked through segment ids; the
+    ~45k-token CogVideoX1.5 joint sequence of Table 3): each sample is
+    text_slots text tokens followed by the video tokens; a sample's valid text
+    length is uniform on the inclusive range [lo, hi]; segment id 1 marks the
+    valid text and every video token, 0 the padded text slots, for queries
+    and keys alike (self-attention over one sequence).
+Independent streams (lengths, outliers, row subsets, joint text lengths) come from
 SeedSequence(seed).spawn so that adding one never shifts another.
 """
 from __future__ import annotations
@@ -53,6 +60,7 @@ class Workload:
     outlier_frac: float = 0.0     # fraction of K rows multiplied by 8
     kv_len_range: tuple | None = None   # inclusive (lo, hi) per-sample text lengths
     oracle_rows: int | None = None      # per (b, h) query rows the parity check compares
+    joint_text: tuple | None = None     # (text_slots, lo, hi): joint text-video segments
     description: str = field(default="", compare=False)
 
     @property
@@ -62,6 +70,10 @@ class Workload:
     @property
     def varlen(self) -> bool:
         return self.kv_len_range is not None
+
+    @property
+    def segments(self) -> bool:
+        return self.joint_text is not None
 
     def flops(self, kv_lens=None) -> float:
         """Algorithmic FLOPs 4*B*H*Sq*Skv*D (two GEMMs, 2 flops per MAC).
@@ -93,13 +105,18 @@ WORKLOADS = {
         "large720", B=1, H=40, D=128, Sq=75600, Skv=75600, seed=1005, latent=(21, 45, 80),
         oracle_rows=4096,
         description="large-DiT 720p self-attention, latent 21x45x80 -> 75600 tokens"),
+    "joint45k": Workload(
+        "joint45k", B=2, H=48, D=64, Sq=45106, Skv=45106, seed=1006, latent=(11, 48, 85),
+        joint_text=(226, 16, 226), oracle_rows=4096,
+        description="joint text-video self-attention, 226 text slots + latent 11x48x85 = 44880 video "
+                    "tokens, padded text masked by segment ids, CFG batch 2, D=64"),
 }
 
 # The bench's default workload: the small-DiT 480p self-attention.
 DEFAULT_WORKLOAD = "small480"
 
 
-def _spawn(seed: int, n: int = 3):
+def _spawn(seed: int, n: int = 4):
     return [np.random.Generator(np.random.PCG64(s)) for s in np.random.SeedSequence(seed).spawn(n)]
 
 
@@ -146,6 +163,21 @@ def draw_rows(B, H, Sq, n, seed) -> np.ndarray:
     return np.stack([np.sort(rng.choice(Sq, size=n, replace=False)) for _ in range(B * H)]).astype(np.int32)
 
 
+def draw_text_lens(B, lo, hi, seed) -> np.ndarray:
+    """Per-sample valid text lengths of a joint sequence, uniform on [lo, hi]."""
+    rng = _spawn(seed)[3]
+    return rng.integers(lo, hi + 1, size=B, dtype=np.int64).astype(np.int32)
+
+
+def joint_segments(text_lens, text_slots, S) -> np.ndarray:
+    """Segment ids [B, S] int32 of joint sequences: text_slots text tokens, then
+    video tokens; 1 for valid text and video, 0 for padded text slots."""
+    seg = np.ones((len(text_lens), S), dtype=np.int32)
+    for b, L in enumerate(np.asarray(text_lens)):
+        seg[b, int(L):text_slots] = 0
+    return seg
+
+
 def pad_invalid_keys(k: torch.Tensor, v: torch.Tensor, kv_lens, fill_bits: int = BF16_NAN_BITS):
     """Overwrite K/V rows past each sample's valid length with a bf16 bit pattern."""
     k = k.clone()
@@ -165,7 +197,8 @@ def generate(w: Workload | str, nan_padding: bool = True):
 
     Returns a dict with q, k, v (bf16 CPU tensors [B,H,S,D]), scale,
     kv_lens (int32 numpy [B] or None), rows (int32 [B*H, n] or None: the
-    query rows a parity check compares) and the workload itself.
+    query rows a parity check compares), q_seg / kv_seg (int32 numpy
+    [B,Sq] / [B,Skv] segment ids, or None) and the workload itself.
     """
     if isinstance(w, str):
         w = WORKLOADS[w]
@@ -178,8 +211,13 @@ def generate(w: Workload | str, nan_padding: bool = True):
         kv_lens = draw_kv_lens(w.B, w.kv_len_range[0], w.kv_len_range[1], w.seed)
         if nan_padding:
             k, v = pad_invalid_keys(k, v, kv_lens)
+    q_seg = kv_seg = None
+    if w.joint_text is not None:
+        slots, lo, hi = w.joint_text
+        seg = joint_segments(draw_text_lens(w.B, lo, hi, w.seed), slots, w.Sq)
+        q_seg = kv_seg = seg
     rows = None
     if w.oracle_rows is not None and w.oracle_rows < w.Sq:
         rows = draw_rows(w.B, w.H, w.Sq, w.oracle_rows, w.seed)
     return {"workload": w, "q": q, "k": k, "v": v, "scale": w.scale,
-            "kv_lens": kv_lens, "rows": rows}
+            "kv_lens": kv_lens, "rows": rows, "q_seg": q_seg, "kv_seg": kv_seg}

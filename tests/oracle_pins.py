@@ -15,6 +15,10 @@ Sources of the facts (none of them is the oracle's own code):
   * masking: a sample with L valid keys equals dense attention on the first
     L keys, whatever the padding holds (appendix Table 4 of the paper:
     padded text tokens must not be attended);
+  * segment ids (joint text-video attention, same appendix entry): one
+    segment everywhere is dense attention; packed segments are independent
+    problems; a prefix segment is the valid-count form; torch's SDPA with the
+    boolean mask q_seg[i] == kv_seg[j];
   * torch's scaled_dot_product_attention and logsumexp in fp64 (a library);
   * a 50-digit mpmath evaluation on a tiny input.
 """
@@ -226,7 +230,82 @@ def pin_large_logits_stable(orc):
         np.testing.assert_allclose(lse[0, 0, 0], want_lse, rtol=1e-15, atol=0)
 
 
+def pin_segments_one_segment_is_dense(orc):
+    """Every query and key in one segment (any id): exactly dense attention."""
+    q, k, v = _inputs(2, 2, 9, 14, 16, seed=26, gain=1.5)
+    o, lse = orc.attn_fwd(q, k, v, 0.3)
+    for sid in (0, 7, -4):
+        os_, ls = orc.attn_fwd(q, k, v, 0.3, q_seg=np.full((2, 9), sid), kv_seg=np.full((2, 14), sid))
+        np.testing.assert_array_equal(os_, o)
+        np.testing.assert_array_equal(ls, lse)
+
+
+def pin_segments_packed_are_independent(orc):
+    """Sequences packed into one with distinct segment ids equal separate attention
+    over each sequence; a query segment with no key gets o = 0, lse = -inf."""
+    B, H, S, D = 2, 2, 15, 8
+    q, k, v = _inputs(B, H, S, S, D, seed=27, gain=1.3)
+    seg = np.array([[3] * 4 + [5] * 6 + [9] * 5,
+                    [1] * 11 + [2] * 4], dtype=np.int32)
+    q_seg = seg.copy()
+    q_seg[1, 13] = 8          # this query's segment owns no key
+    o, lse = orc.attn_fwd(q, k, v, 0.45, q_seg=q_seg, kv_seg=seg)
+    for b in range(B):
+        for sid in np.unique(seg[b]):
+            js = np.flatnonzero(seg[b] == sid)
+            lo, hi = js[0], js[-1] + 1
+            ob, lb = orc.attn_fwd(q[b:b + 1, :, lo:hi], k[b:b + 1, :, lo:hi], v[b:b + 1, :, lo:hi], 0.45)
+            rows = [i for i in range(lo, hi) if q_seg[b, i] == sid]
+            np.testing.assert_allclose(o[b][:, rows], ob[0][:, np.array(rows) - lo], rtol=0, atol=1e-14)
+            np.testing.assert_allclose(lse[b][:, rows], lb[0][:, np.array(rows) - lo], rtol=1e-15, atol=1e-14)
+    assert np.all(o[1, :, 13] == 0) and np.all(np.isneginf(lse[1, :, 13]))
+
+
+def pin_segments_prefix_is_valid_count(orc):
+    """kv_seg = 1 on the first L keys and 0 after (NaN padding), q_seg = 1:
+    exactly the valid-count form with kv_lens = L."""
+    B, H, Sq, Skv, D = 3, 2, 5, 19, 16
+    q, k, v = random_qkv(B, H, Sq, Skv, D, seed=28, logit_gain=1.4)
+    lens = np.array([19, 6, 1], dtype=np.int32)
+    kp, vp = pad_invalid_keys(k, v, lens)
+    kv_seg = (np.arange(Skv)[None, :] < lens[:, None]).astype(np.int32)
+    q_seg = np.ones((B, Sq), dtype=np.int32)
+    o, lse = orc.attn_fwd(bf16_bits(q), bf16_bits(kp), bf16_bits(vp), 0.25, q_seg=q_seg, kv_seg=kv_seg)
+    ov, lv = orc.attn_fwd(bf16_bits(q), bf16_bits(kp), bf16_bits(vp), 0.25, kv_lens=lens)
+    assert np.all(np.isfinite(o))
+    np.testing.assert_array_equal(o, ov)
+    np.testing.assert_array_equal(lse, lv)
+
+
+def pin_segments_torch_masked_sdpa(orc):
+    """Interleaved segment ids against torch SDPA with the boolean mask
+    q_seg[i] == kv_seg[j] and a masked logsumexp, fp64 (a library)."""
+    B, H, Sq, Skv, D, scale = 2, 3, 21, 26, 32, 0.2
+    q, k, v = random_qkv(B, H, Sq, Skv, D, seed=29, logit_gain=1.6)
+    rng = np.random.default_rng(30)
+    q_seg = rng.integers(0, 3, size=(B, Sq)).astype(np.int32)
+    kv_seg = rng.integers(0, 3, size=(B, Skv)).astype(np.int32)
+    kv_seg[1, :] = np.where(kv_seg[1, :] == 2, 1, kv_seg[1, :])   # sample 1: segment 2 owns no key
+    o, lse, p = orc.attn_fwd(bf16_bits(q), bf16_bits(k), bf16_bits(v), scale, probs=True,
+                             q_seg=q_seg, kv_seg=kv_seg)
+    mask = torch.from_numpy(q_seg[:, :, None] == kv_seg[:, None, :])[:, None]    # [B,1,Sq,Skv]
+    qd, kd, vd = q.double(), k.double(), v.double()
+    want = torch.nn.functional.scaled_dot_product_attention(qd, kd, vd, attn_mask=mask, scale=scale)
+    logits = (scale * (qd @ kd.transpose(-1, -2))).masked_fill(~mask, -math.inf)
+    want_lse = torch.logsumexp(logits, dim=-1)
+    has = mask.numpy().any(-1)                                                   # [B,1,Sq]
+    has = np.broadcast_to(has, (B, H, Sq))
+    assert (~has).any() and has.any()
+    np.testing.assert_allclose(o[has], want.numpy()[has], rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lse[has], want_lse.numpy()[has], rtol=1e-13, atol=1e-12)
+    assert np.all(o[~has] == 0) and np.all(np.isneginf(lse[~has]))
+    np.testing.assert_array_equal(p == 0, ~np.broadcast_to(mask.numpy(), p.shape) | (p == 0))
+    np.testing.assert_allclose(p.sum(-1)[has], 1.0, rtol=0, atol=1e-13)
+
+
 ALL_PINS = [pin_single_key, pin_two_keys, pin_weights_sum_to_one, pin_constant_values,
             pin_zero_logits, pin_query_permutation, pin_key_value_permutation,
             pin_value_translation, pin_varlen_is_truncation, pin_varlen_empty_and_clamped,
-            pin_row_subset, pin_torch_sdpa, pin_mpmath_brute_force, pin_large_logits_stable]
+            pin_row_subset, pin_torch_sdpa, pin_mpmath_brute_force, pin_large_logits_stable,
+            pin_segments_one_segment_is_dense, pin_segments_packed_are_independent,
+            pin_segments_prefix_is_valid_count, pin_segments_torch_masked_sdpa]

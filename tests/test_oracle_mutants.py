@@ -18,7 +18,7 @@ SOURCE = os.path.join(ROOT, "oracle", "oracle.c")
 MUTANTS = {
     "scale_dropped": [("s[j] = scale * dot;", "s[j] = dot;")],
     "scale_twice": [("s[j] = scale * dot;", "s[j] = scale * scale * dot;")],
-    "k_transposed": [("bf16_to_f64(k[(size_t)j * D + d])", "bf16_to_f64(k[(size_t)d * L + j])")],
+    "k_transposed": [("bf16_to_f64(k[kj * D + d])", "bf16_to_f64(k[(size_t)d * L + kj])")],
     "dot_skips_first_dim": [("for (int d = 0; d < D; ++d)\n            dot",
                              "for (int d = 1; d < D; ++d)\n            dot")],
     "lse_drops_max": [("*lse = m + log(l);", "*lse = log(l);")],
@@ -27,13 +27,22 @@ MUTANTS = {
     "no_max_shift": [("exp(s[j] - m)", "exp(s[j])"), ("*lse = m + log(l);", "*lse = log(l);")],
     "min_not_max": [("if (s[j] > m)", "if (s[j] < m)")],
     "not_normalised": [("double p = exp(s[j] - m) / l;", "double p = exp(s[j] - m);")],
-    "v_dims_reversed": [("bf16_to_f64(v[(size_t)j * D + d])", "bf16_to_f64(v[(size_t)j * D + (D - 1 - d)])")],
+    "v_dims_reversed": [("bf16_to_f64(v[vj * D + d])", "bf16_to_f64(v[vj * D + (D - 1 - d)])")],
     "varlen_off_by_one": [("int L = kv_lens[b];", "int L = kv_lens[b] + 1;")],
     "varlen_wrong_sample": [("valid_len(kv_lens, b, Skv)", "valid_len(kv_lens, 0, Skv)")],
     "rows_ignore_head": [("rows[bh * nrows + r]", "rows[r]")],
     "q_ignores_head": [("((size_t)bh * Sq + i) * D", "((size_t)i) * D")],
     "k_ignores_head": [("k + (size_t)bh * Skv * D", "k")],
     "v_ignores_head": [("v + (size_t)bh * Skv * D", "v")],
+    "seg_not_equal": [("if (kseg[j] == seg)", "if (kseg[j] != seg)")],
+    "seg_keys_of_sample_0": [("kv_seg + (size_t)b * Skv", "kv_seg")],
+    "seg_first_query_id": [("q_seg[(size_t)b * Sq + i]", "q_seg[(size_t)b * Sq]")],
+    "seg_query_ids_of_sample_0": [("q_seg[(size_t)b * Sq + i]", "q_seg[i]")],
+    "seg_drops_last_key": [("for (int j = 0; j < Skv; ++j)\n                if (kseg",
+                            "for (int j = 0; j < Skv - 1; ++j)\n                if (kseg")],
+    "seg_k_by_position": [("const size_t kj = (size_t)(idx ? idx[j] : j);", "const size_t kj = (size_t)j;")],
+    "seg_v_by_position": [("const size_t vj = (size_t)(idx ? idx[j] : j);", "const size_t vj = (size_t)j;")],
+    "seg_probs_by_position": [("pr[idx[e]] = ps[e];", "pr[e] = ps[e];")],
 }
 
 CHILD = r"""
