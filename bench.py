@@ -2,11 +2,12 @@
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
 
-One step = one attention forward (one vdx_attn_fwd / vdx_attn_fwd_varlen
-launch) over the whole workload, inputs resident in HBM.  The default
-workload is the small-DiT 480p self-attention (B=1, H=12, D=128,
-S = 21*30*52 = 32760 tokens, logit std ~3).  FLOPs = 4*B*H*Sq*Skv*D
-(effective key counts for the padded-text workload).
+One step = one attention forward (one vdx_attn_fwd / vdx_attn_fwd_varlen /
+vdx_attn_fwd_segments call) over the whole workload, inputs resident in
+HBM.  The default workload is the small-DiT 480p self-attention (B=1, H=12,
+D=128, S = 21*30*52 = 32760 tokens, logit std ~3).  FLOPs = 4*B*H*Sq*Skv*D
+(effective key counts for the padded-text workload; the (query, key) pairs
+of equal segment id for the joint text-video workload).
 
 Timing: W untimed warm-up steps, then K steps bracketed by a barrier and a
 device synchronisation, timed with CUDA events on the launching stream; the
@@ -129,7 +130,7 @@ class ClockSampler:
 def make_inputs(name):
     from paper_2609_18077_gb300 import workloads
     w = workloads.generate(name)
-    flops = w["workload"].flops(w["kv_lens"])
+    flops = w["workload"].flops(w["kv_lens"], w["q_seg"], w["kv_seg"])
     return w, flops
 
 
@@ -148,12 +149,18 @@ def run_ours(args):
     wl = w["workload"]
     q, k, v = (t.to(dev) for t in (w["q"], w["k"], w["v"]))
     lens = None if w["kv_lens"] is None else torch.from_numpy(w["kv_lens"]).to(dev)
+    segs = None if w["q_seg"] is None else tuple(torch.from_numpy(w[n]).to(dev) for n in ("q_seg", "kv_seg"))
     out = torch.empty_like(q)
     lse = torch.empty(q.shape[:3], dtype=torch.float32, device=dev)
     stream = torch.cuda.current_stream(dev)
+    # kernels of ours per step: the segment path builds its key-tile lists first
+    launches_per_step = 3 if segs is not None else 1
+    mode = "seg" if segs is not None else ("varlen" if lens is not None else "dense")
 
     def step():
-        if lens is None:
+        if segs is not None:
+            binding.attn_fwd_segments(q, k, v, segs[0], segs[1], scale=wl.scale, out=out, lse=lse)
+        elif lens is None:
             binding.attn_fwd(q, k, v, scale=wl.scale, out=out, lse=lse)
         else:
             binding.attn_fwd_varlen(q, k, v, lens, scale=wl.scale, out=out, lse=lse)
@@ -192,9 +199,11 @@ def run_ours(args):
     # ---- end to end through the C ABI with pinned host buffers
     qh, kh, vh = (t.pin_memory() for t in (w["q"], w["k"], w["v"]))
     lh = None if w["kv_lens"] is None else torch.from_numpy(w["kv_lens"]).pin_memory()
+    sh = None if segs is None else tuple(torch.from_numpy(w[n]).pin_memory() for n in ("q_seg", "kv_seg"))
     oh = torch.empty(out.shape, dtype=out.dtype).pin_memory()
     lseh = torch.empty(lse.shape, dtype=lse.dtype).pin_memory()
-    h2d = sum(t.numel() * t.element_size() for t in (qh, kh, vh)) + (0 if lh is None else lh.numel() * 4)
+    h2d = sum(t.numel() * t.element_size() for t in (qh, kh, vh)) + (0 if lh is None else lh.numel() * 4) + \
+        (0 if sh is None else sum(t.numel() * 4 for t in sh))
     d2h = oh.numel() * oh.element_size() + lseh.numel() * lseh.element_size()
 
     def e2e_step():
@@ -203,6 +212,9 @@ def run_ours(args):
         v.copy_(vh, non_blocking=True)
         if lh is not None:
             lens.copy_(lh, non_blocking=True)
+        if sh is not None:
+            segs[0].copy_(sh[0], non_blocking=True)
+            segs[1].copy_(sh[1], non_blocking=True)
         step()
         oh.copy_(out, non_blocking=True)
         lseh.copy_(lse, non_blocking=True)
@@ -247,14 +259,13 @@ def run_ours(args):
         "clocks": clocks,
         "e2e": {"value": round(e2e_tflops, 2), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
-        "gpu_launches": args.steps,
+        "gpu_launches": args.steps * launches_per_step,
         "roofline": {"bound": "tensor", "achieved": round(per_launch_tflops, 2), "peak": peak,
                      "unit": "TFLOP/s", "frac": round(per_launch_tflops / peak, 4),
                      "peak_kind": f"{peak_kind} bf16 dense burst",
                      "frac_of_sustained": round(per_launch_tflops / float(peaks["bf16_tflops_sustained"]), 4),
                      "traffic": traffic,
-                     "kernel": "vdx::attn_fwd_kernel<%d,%s,%s>" % (wl.D, "true" if lens is not None else "false",
-                                                                      "1,2" if wl.D == 128 else "2,4")},
+                     "kernel": "vdx::attn_fwd_kernel<%d,%s,%s>" % (wl.D, mode, "1,2" if wl.D == 128 else "2,4")},
         "cpu_baseline": cpu,
     }
     print(json.dumps(line), flush=True)
@@ -305,6 +316,8 @@ class OracleTimer:
         self.rng = np.random.default_rng(wl.seed)
         lens = w["kv_lens"]
         keys = wl.Skv if lens is None else float(np.mean(np.clip(lens, 0, wl.Skv)))
+        if w["q_seg"] is not None:   # mean keys per query row
+            keys = workloads.segment_pairs(w["q_seg"], w["kv_seg"]) / float(wl.B * wl.Sq)
         self.flops_per_row = 4.0 * keys * wl.D
         self.bh = wl.B * wl.H
         self.n = 1
@@ -313,7 +326,8 @@ class OracleTimer:
         rows = np.stack([np.sort(self.rng.choice(self.wl.Sq, size=n, replace=False))
                          for _ in range(self.bh)]).astype(np.int32)
         t0 = time.perf_counter()
-        self.orc.attn_fwd(*self.bits, self.wl.scale, kv_lens=self.w["kv_lens"], rows=rows)
+        self.orc.attn_fwd(*self.bits, self.wl.scale, kv_lens=self.w["kv_lens"], rows=rows,
+                          q_seg=self.w["q_seg"], kv_seg=self.w["kv_seg"])
         return time.perf_counter() - t0
 
     def calibrate(self, target_s):

@@ -10,13 +10,17 @@
  *     sample, so attention cost is quadratic in the token count;
  *   - appendix Table 4 (porting-bug taxonomy): padded text tokens must be
  *     excluded, by skipping invalid key blocks rather than by a dense
- *     (B, H, Sq, Sk) mask -- the varlen entry point below.
+ *     (B, H, Sq, Sk) mask -- the varlen entry point below, and its
+ *     generalisation to per-token segment ids for joint text-video
+ *     attention (HunyuanVideo-1.5 in that entry; the ~45k-token CogVideoX1.5
+ *     joint sequence of Table 3) -- vdx_attn_fwd_segments.
  *
- * For each batch b, head h and query row i, with L valid keys:
- *     s_j  = scale * <q[b,h,i,:], k[b,h,j,:]>,            j < L
+ * For each batch b, head h and query row i, over its valid keys j (the first
+ * L of them, or those of its segment):
+ *     s_j  = scale * <q[b,h,i,:], k[b,h,j,:]>
  *     out[b,h,i,:] = sum_j softmax(s)_j * v[b,h,j,:]
  *     lse[b,h,i]   = ln(sum_j exp(s_j))                  (natural log)
- * L = 0 gives out = 0 and lse = -inf.
+ * No valid key gives out = 0 and lse = -inf.
  *
  * Conventions shared by every entry point:
  *   - Tensors are contiguous, row-major, bf16 (IEEE bfloat16 bits):
@@ -27,7 +31,9 @@
  *     multiprocessors idle (dense calls only), the library splits those units
  *     along the keys and merges the parts through a device workspace of
  *     (tail units x parts x 2 x 128 x (D + 4)) fp32 values -- about 19 MB for
- *     B=1, H=12, S=32760, D=128.  The workspace belongs to the library, one per
+ *     B=1, H=12, S=32760, D=128.  Segment calls keep their key-tile lists in
+ *     the same workspace: B x ceil(Sq/256) x ceil(Skv/128) x 4 bytes plus
+ *     ranges (about 0.5 MB for B=2, S=45106).  The workspace belongs to the library, one per
  *     (device, stream): it is allocated by the first call that needs it, grown
  *     by a later call that needs more (that call waits for the device), and
  *     kept until the process exits.  Calls on the same stream share it in
@@ -80,6 +86,26 @@ int vdx_attn_fwd(const void *q, const void *k, const void *v, void *out, float *
 int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, float *lse,
                         int B, int H, int Sq, int Skv_max, int D, const int *kv_lens,
                         float scale, void *stream);
+
+/*
+ * Joint attention with segment ids (appendix Table 4: padded text tokens in
+ * a joint text-video sequence are masked through segment ids so that the
+ * kernel skips invalid key blocks).  As vdx_attn_fwd, except that query i of
+ * sample b attends exactly the keys j with kv_seg[b*Skv + j] == q_seg[b*Sq + i].
+ *   q_seg : DEVICE int32 [B, Sq],  kv_seg : DEVICE int32 [B, Skv], caller-owned,
+ *           4-byte aligned, shared by all heads; any int32 values.
+ * A query whose segment owns no key gets out = 0 and lse = -inf.  Key tiles
+ * (128 keys) holding no id of a query tile pair's range are skipped; tiles
+ * holding one id equal to the query tile's single id run unmasked; the rest
+ * compare ids element by element.  Every V row must be finite: a key of
+ * another segment inside a visited tile enters the tensor-core product with
+ * weight exactly 0, and 0 x NaN = NaN (K may hold any bits there).
+ * Two small kernels build the key-tile lists before the attention kernel, on
+ * the same stream, in the library's per-stream workspace (see Memory above).
+ */
+int vdx_attn_fwd_segments(const void *q, const void *k, const void *v, void *out, float *lse,
+                          int B, int H, int Sq, int Skv, int D, const int *q_seg, const int *kv_seg,
+                          float scale, void *stream);
 
 /*
  * vdx_attn_fwd without any device allocation (the paper has no counterpart;

@@ -31,6 +31,7 @@ _I = ctypes.c_int
 SIGNATURES = {
     "vdx_attn_fwd": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, ctypes.c_float, _P]),
     "vdx_attn_fwd_varlen": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, ctypes.c_float, _P]),
+    "vdx_attn_fwd_segments": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, ctypes.c_float, _P]),
     "vdx_attn_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, ctypes.c_float, _P]),
     "vdx_status_string": (ctypes.c_char_p, [_I]),
     "vdx_check_device_error": (_I, [_P]),
@@ -155,4 +156,29 @@ def attn_fwd_varlen(q, k, v, kv_lens, scale=None, out=None, lse=None, return_lse
                                         _stream_handle(q.device))
     if st != VDX_OK:
         raise VdxError(st, "vdx_attn_fwd_varlen")
+    return out, lse
+
+
+def attn_fwd_segments(q, k, v, q_seg, kv_seg, scale=None, out=None, lse=None, return_lse=True):
+    """Joint attention with segment ids through ``vdx_attn_fwd_segments``.
+
+    q_seg: int32 CUDA tensor [B, Sq]; kv_seg: int32 CUDA tensor [B, Skv]; query i
+    of sample b attends the keys j with kv_seg[b, j] == q_seg[b, i].
+    """
+    _check_qkv(q, k, v)
+    B, H, Sq, D = q.shape
+    Skv = k.shape[2]
+    for name, t, n in (("q_seg", q_seg, Sq), ("kv_seg", kv_seg, Skv)):
+        if (not isinstance(t, torch.Tensor) or t.dtype != torch.int32 or tuple(t.shape) != (B, n)
+                or t.device != q.device or not t.is_contiguous()):
+            raise TypeError(f"{name} must be a contiguous int32 CUDA tensor of shape [{B}, {n}] on q's device")
+    scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
+    out, lse = _outputs(q, out, lse, return_lse)
+    with torch.cuda.device(q.device):
+        st = load().vdx_attn_fwd_segments(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                                          lse.data_ptr() if lse is not None else None,
+                                          B, H, Sq, Skv, D, q_seg.data_ptr(), kv_seg.data_ptr(), scale,
+                                          _stream_handle(q.device))
+    if st != VDX_OK:
+        raise VdxError(st, "vdx_attn_fwd_segments")
     return out, lse

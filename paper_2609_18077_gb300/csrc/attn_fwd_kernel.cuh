@@ -6,7 +6,11 @@
 // log-sum-exp, without ever storing the Sq x Skv score matrix, over
 // [B, H, S, D] bf16 video tokens.  The varlen instance skips key tiles past a
 // sample's valid text length and masks the ragged last tile (appendix Table 4:
-// segment-id masking of padded text keys instead of a dense mask).
+// segment-id masking of padded text keys instead of a dense mask).  The
+// segment instance (joint text-video attention, same appendix entry) lets
+// query i attend key j iff their segment ids match: each unit visits only the
+// key tiles of its list (segment_tiles.cuh) and compares ids element by
+// element only on the tiles the list marks.
 //
 // Work unit: one (b*h, pair of 128-row query tiles).  The grid is persistent:
 // one CTA per SM walks the units u = blockIdx.x, blockIdx.x + gridDim.x, ...
@@ -54,9 +58,15 @@
 #include <cuda_bf16.h>
 #include <cstdint>
 
+#include "segment_tiles.cuh"
 #include "sm103_ptx.cuh"
 
 namespace vdx {
+
+// Problem kinds (template parameter MODE of the kernel).
+constexpr int MODE_DENSE = 0;    // all Skv keys
+constexpr int MODE_VARLEN = 1;   // the first kv_lens[b] keys of sample b
+constexpr int MODE_SEG = 2;      // the keys whose segment id equals the query's
 
 // Device error word: bit 0 = a bounded wait expired.  Read and cleared by
 // vdx_check_device_error.
@@ -93,6 +103,19 @@ struct AttnParams {
     uint64_t wait_limit_ns;
 };
 
+// Segment ids (MODE_SEG): q_seg [B, Sq], kv_seg [B, Skv]; per (b, query-tile
+// pair) the key-tile list tlist[(b * q_pairs + qp) * n_kt + r], r < tcount[.].
+// A kernel parameter of its own: with these fields inside AttnParams the
+// register allocation of the dense and varlen kernels changed and the dense
+// kernel measured 2 % slower.
+struct SegParams {
+    const int *q_seg;
+    const int *kv_seg;
+    const uint32_t *tlist;
+    const int *tcount;
+    int n_kt;             // key tiles of the whole sequence, ceil(Skv / BN)
+};
+
 // Shared-memory plan.  QBUF Q-tile pairs (2 = the next item's Q tiles load
 // while the current item runs) and NSTAGE K/V stages of (V_j, next K).
 template <int D, int QBUF, int NSTAGE_>
@@ -120,6 +143,8 @@ struct Layout {
     static constexpr int TMEM_PTR_OFF = BAR_OFF + NBARS * 8;
     static constexpr int ABORT_OFF = TMEM_PTR_OFF + 4;
     static constexpr int MERGE_OFF = ABORT_OFF + 4;          // "this CTA merges" flag
+    // 197.8 KB in all configurations: under the 196 KB shared-memory carve-out
+    // (199,680 usable bytes), which leaves 60 KB of L1 for the spill slots.
     static constexpr int BYTES = MERGE_OFF + 4;
     static constexpr int ALLOC = BYTES + 1024;               // slack for 1024-B alignment
 };
@@ -352,30 +377,38 @@ __device__ __noinline__ void merge_tail_parts(const AttnParams &p, int tail, int
 
 // One work item of a CTA: a whole unit (b*h, query-tile pair) with key tiles
 // [j0, j1) = [0, n_kv), or -- for the units of a short last round, when the
-// host splits them -- one part of such a unit's key tiles (part >= 0).
+// host splits them -- one part of such a unit's key tiles (part >= 0).  In
+// MODE_SEG, j indexes the unit's key-tile list rather than the key tiles.
 struct Item {
     int bh;
     int qp;
     int kv_valid;
-    int n_kv;      // key tiles of the whole unit
+    int n_kv;      // key tiles of the whole unit (MODE_SEG: list entries)
     int j0, j1;    // key tiles of this item
     int part;      // -1: whole unit; else the part index within tail unit `tail`
     int tail;
+    int list_off;  // MODE_SEG: offset of the unit's list in tlist
     bool ok;       // false past the CTA's last item
 };
 
-template <bool VARLEN>
-__device__ __forceinline__ Item unit_item(const AttnParams &p, int u)
+template <int MODE>
+__device__ __forceinline__ Item unit_item(const AttnParams &p, const SegParams &sp, int u)
 {
     Item w;
     w.bh = u / p.q_pairs;
     w.qp = u - w.bh * p.q_pairs;
     w.kv_valid = p.Skv;
-    if (VARLEN) {
+    w.list_off = 0;
+    if (MODE == MODE_VARLEN) {
         const int len = __ldg(p.kv_lens + w.bh / p.H);
         w.kv_valid = len < 0 ? 0 : (len > p.Skv ? p.Skv : len);
     }
     w.n_kv = (w.kv_valid + BN - 1) / BN;
+    if (MODE == MODE_SEG) {
+        const int pair = (w.bh / p.H) * p.q_pairs + w.qp;
+        w.n_kv = __ldg(sp.tcount + pair);
+        w.list_off = pair * sp.n_kt;
+    }
     w.j0 = 0;
     w.j1 = w.n_kv;
     w.part = -1;
@@ -386,8 +419,8 @@ __device__ __forceinline__ Item unit_item(const AttnParams &p, int u)
 
 // The i-th item of CTA `cta`: units cta, cta + G, ... and, in split mode,
 // after full_rounds of them one part of a tail unit.
-template <bool VARLEN>
-__device__ __forceinline__ Item item_at(const AttnParams &p, int cta, int i)
+template <int MODE>
+__device__ __forceinline__ Item item_at(const AttnParams &p, const SegParams &sp, int cta, int i)
 {
     const int G = gridDim.x;
     Item w;
@@ -395,15 +428,15 @@ __device__ __forceinline__ Item item_at(const AttnParams &p, int cta, int i)
     if (p.split_parts == 0) {
         const int u = cta + i * G;
         if (u < p.units)
-            w = unit_item<VARLEN>(p, u);
+            w = unit_item<MODE>(p, sp, u);
         return w;
     }
     if (i < p.full_rounds)
-        return unit_item<VARLEN>(p, cta + i * G);
+        return unit_item<MODE>(p, sp, cta + i * G);
     if (i == p.full_rounds && cta < p.tail_units * p.split_parts) {
         const int tail = cta / p.split_parts;
         const int part = cta - tail * p.split_parts;
-        w = unit_item<VARLEN>(p, p.full_rounds * G + tail);
+        w = unit_item<MODE>(p, sp, p.full_rounds * G + tail);
         w.j0 = part * w.n_kv / p.split_parts;
         w.j1 = (part + 1) * w.n_kv / p.split_parts;
         w.part = part;
@@ -412,10 +445,20 @@ __device__ __forceinline__ Item item_at(const AttnParams &p, int cta, int i)
     return w;
 }
 
-template <int D, bool VARLEN, int QBUF, int NSTAGE>
+// Key tile of list position r of item w (the identity unless MODE_SEG).
+template <int MODE>
+__device__ __forceinline__ int key_tile(const SegParams &sp, const Item &w, int r)
+{
+    if (MODE == MODE_SEG)
+        return static_cast<int>(__ldg(sp.tlist + w.list_off + r) & SEG_TILE_BITS);
+    return r;
+}
+
+template <int D, int MODE, int QBUF, int NSTAGE>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
-                    const __grid_constant__ CUtensorMap tmap_v, const AttnParams p)
+                    const __grid_constant__ CUtensorMap tmap_v, const AttnParams p,
+                    const __grid_constant__ SegParams sp)
 {
     using L = Layout<D, QBUF, NSTAGE>;
     extern __shared__ uint8_t smem_raw[];
@@ -473,7 +516,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // holds that first key tile alone.
         auto next_with_keys = [&](int i) {
             for (++i;; ++i) {
-                const Item w = item_at<VARLEN>(p, cta, i);
+                const Item w = item_at<MODE>(p, sp, cta, i);
                 if (!w.ok)
                     return -1;
                 if (w.j1 > w.j0)
@@ -494,7 +537,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const uint32_t vdst = sbase + L::KV_OFF + (2 * st) * L::TILE_BYTES;
             const uint32_t kdst = vdst + L::TILE_BYTES;
             const bool has_v = vj >= 0, has_k = kj >= 0;
-            const bool fix = VARLEN && has_v && v_valid < BN;
+            const bool fix = MODE == MODE_VARLEN && has_v && v_valid < BN;
             if (fix) {
                 // A padded sample's last V tile: rows past the valid length may
                 // hold any bits (NaN included) and 0 * NaN = NaN inside the
@@ -538,18 +581,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         };
         int i = 0;
         {
-            const Item w0 = item_at<VARLEN>(p, cta, 0);
+            const Item w0 = item_at<MODE>(p, sp, cta, 0);
             if (!w0.ok)
                 i = -1;
             else if (w0.j1 == w0.j0)
                 i = next_with_keys(0);
         }
         if (i >= 0) {
-            const Item w = item_at<VARLEN>(p, cta, i);
-            ok = stage(0, -1, BN, w.bh, w.j0);
+            const Item w = item_at<MODE>(p, sp, cta, i);
+            ok = stage(0, -1, BN, w.bh, key_tile<MODE>(sp, w, w.j0));
         }
         for (int iq = 0; ok && i >= 0; ++iq) {
-            const Item w = item_at<VARLEN>(p, cta, i);
+            const Item w = item_at<MODE>(p, sp, cta, i);
             const int ni = next_with_keys(i);
             const int qb = iq % QBUF;
             if (iq >= QBUF) {
@@ -571,12 +614,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             Item nw;
             nw.ok = false;
             if (ni >= 0)
-                nw = item_at<VARLEN>(p, cta, ni);
+                nw = item_at<MODE>(p, sp, cta, ni);
+            int vj = key_tile<MODE>(sp, w, w.j0);
             for (int j = w.j0; ok && j < w.j1; ++j) {
                 const bool last = j + 1 == w.j1;
                 const int kbh = last ? (nw.ok ? nw.bh : 0) : w.bh;
-                const int kj = last ? (nw.ok ? nw.j0 : -1) : j + 1;
-                ok = stage(w.bh, j, w.kv_valid - j * BN, kbh, kj);
+                // MODE_SEG: the list entry is read before the stage's empty wait
+                const int kj = last ? (nw.ok ? key_tile<MODE>(sp, nw, nw.j0) : -1) : key_tile<MODE>(sp, w, j + 1);
+                ok = stage(w.bh, vj, w.kv_valid - vj * BN, kbh, kj);
+                vj = kj;
             }
             i = ni;
         }
@@ -594,7 +640,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             int iq = 0;        // items with keys so far
             bool ok = true;
             for (int i = 0; ok; ++i) {
-                const Item w = item_at<VARLEN>(p, cta, i);
+                const Item w = item_at<MODE>(p, sp, cta, i);
                 if (!w.ok)
                     break;
                 const int n = w.j1 - w.j0;
@@ -688,7 +734,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         bool ok = true;
 
         for (int i = 0; ok; ++i) {
-            const Item w = item_at<VARLEN>(p, cta, i);
+            const Item w = item_at<MODE>(p, sp, cta, i);
             if (!w.ok)
                 break;
             const int q_row = (w.qp * 2 + t) * BM + row;
@@ -707,7 +753,35 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             float m_used = -INFINITY;
             float l_exact = 0.f;   // sum of the fp32 weights: the log-sum-exp
             float l_resid = 0.f;   // sum over tiles of r - p for each tile's largest weight
+            // MODE_SEG: this row's segment id, the sample's key ids and the next list entry
+            int my_seg = 0;
+            const int *kseg = nullptr;
+            uint32_t next_entry = 0;
+            if (MODE == MODE_SEG) {
+                const size_t b = static_cast<size_t>(w.bh / p.H);
+                my_seg = store ? __ldg(sp.q_seg + b * p.Sq + q_row) : 0;
+                kseg = sp.kv_seg + b * p.Skv;
+                next_entry = __ldg(sp.tlist + w.list_off + w.j0);
+            }
             for (int j = w.j0; j < w.j1; ++j, ++sc) {
+                int kt = j;   // key tile
+                bool seg_mask = false;
+                int ids[4];
+                if (MODE == MODE_SEG) {
+                    const uint32_t entry = next_entry;
+                    kt = static_cast<int>(entry & SEG_TILE_BITS);
+                    if (j + 1 < w.j1)
+                        next_entry = __ldg(sp.tlist + w.list_off + j + 1);
+                    seg_mask = (entry >> (SEG_MASK_SHIFT + t)) & 1u;
+                    if (seg_mask) {
+                        // this lane's four of the tile's 128 key ids, read under the S wait
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const int c = kt * BN + e * 32 + lane;
+                            ids[e] = c < p.Skv ? __ldg(kseg + c) : 0;
+                        }
+                    }
+                }
                 if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_S + t), sc & 1, abort_flag, limit))))
                     break;
                 ptx::tc_fence_after_sync();
@@ -725,7 +799,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 ptx::tmem_wait_ld();
 
-                const int valid = w.kv_valid - j * BN;
+                const int valid = w.kv_valid - kt * BN;
                 if (valid < BN) {
                     // Ragged last tile: keys past the end (or past the sample's
                     // text length, whatever their bits) become -inf logits
@@ -736,6 +810,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     for (int c = 0; c < BN; ++c)
                         s[c >> 5][c & 31] = c < valid ? s[c >> 5][c & 31] : pad;
                 }
+                if (MODE == MODE_SEG && seg_mask) {
+                    // Keys of another segment get the masked logit too.  Lane
+                    // l holds the ids of keys 32e + l; the warp shares them by
+                    // shuffles (a marked tile is rare: segment borders only).
+                    const uint32_t pad = neg_scale ? 0x7F800000u : 0xFF800000u;
+#pragma unroll
+                    for (int c = 0; c < BN; ++c) {
+                        const int kid = __shfl_sync(0xffffffffu, ids[c >> 5], c & 31);
+                        s[c >> 5][c & 31] = kid == my_seg ? s[c >> 5][c & 31] : pad;
+                    }
+                }
                 const float ext = row_extreme(s, neg_scale);
                 const float m_tile = ext * sl2;
                 const float m_new = fmaxf(m_used, m_tile);
@@ -745,7 +830,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     factor = ex2(m_used - m_new);
                     m_used = m_new;
                 }
-                const float neg_m = -m_used;
+                // MODE_SEG: a row whose keys so far were all masked keeps
+                // m_used = -inf; its weights are 2^-inf = 0, not 2^(-inf + inf).
+                const float neg_m = (MODE == MODE_SEG && m_used == -INFINITY) ? 0.f : -m_used;
                 // the tile's largest weight, computed exactly as in row_probs
                 const float p_top = ex2(fmaf(ext, sl2, neg_m));
                 l_exact *= factor;
@@ -806,7 +893,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                     reinterpret_cast<volatile int *>(sm + L::MERGE_OFF), bar(L::B_MERGE),
                                     bar(L::B_MERGE + 1), abort_flag);
             } else {
-                const float inv_l = 1.f / (l_exact + l_resid);
+                // MODE_SEG: a row with no key of its segment has l = 0 and O = 0.
+                const float inv_l = (MODE == MODE_SEG && !(l_exact > 0.f)) ? 0.f : 1.f / (l_exact + l_resid);
                 uint32_t w16[D / 32][16];
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {

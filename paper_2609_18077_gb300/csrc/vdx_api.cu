@@ -3,8 +3,10 @@
 // Validation happens before any CUDA call; then, once per device, the device
 // is checked to be sm_103 and the kernels' shared-memory limits are raised;
 // then three 3-D TMA tensor maps (head dim, sequence, batch*head) are encoded
-// and one kernel is launched on the caller's stream.  The only allocation is
-// the split-tail workspace (per device and stream, made once, kept).
+// and one kernel is launched on the caller's stream (joint attention with
+// segment ids first launches two small kernels that build its key-tile
+// lists).  The only allocation is the workspace of the split tail and of the
+// key-tile lists (per device and stream, made once, grown, kept).
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -56,10 +58,10 @@ DeviceState g_devices[kMaxDevices];
 // text cross-attention); D = 64 fits two Q buffers (the next item's Q loads a
 // whole item ahead) and four stages.
 
-template <int D, bool VARLEN, int QBUF, int NSTAGE>
+template <int D, int MODE, int QBUF, int NSTAGE>
 cudaError_t raise_smem_limit()
 {
-    return cudaFuncSetAttribute(vdx::attn_fwd_kernel<D, VARLEN, QBUF, NSTAGE>,
+    return cudaFuncSetAttribute(vdx::attn_fwd_kernel<D, MODE, QBUF, NSTAGE>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
                                 vdx::Layout<D, QBUF, NSTAGE>::ALLOC);
 }
@@ -67,19 +69,21 @@ cudaError_t raise_smem_limit()
 cudaError_t raise_all_smem_limits()
 {
     cudaError_t e = cudaSuccess;
-    for (cudaError_t r : {raise_smem_limit<128, false, 1, 2>(), raise_smem_limit<128, true, 1, 2>(),
-                          raise_smem_limit<64, false, 2, 4>(), raise_smem_limit<64, true, 2, 4>()})
+    using namespace vdx;
+    for (cudaError_t r : {raise_smem_limit<128, MODE_DENSE, 1, 2>(), raise_smem_limit<128, MODE_VARLEN, 1, 2>(),
+                          raise_smem_limit<128, MODE_SEG, 1, 2>(), raise_smem_limit<64, MODE_DENSE, 2, 4>(),
+                          raise_smem_limit<64, MODE_VARLEN, 2, 4>(), raise_smem_limit<64, MODE_SEG, 2, 4>()})
         if (r != cudaSuccess)
             e = r;
     return e;
 }
 
-template <int D, bool VARLEN, int QBUF, int NSTAGE>
+template <int D, int MODE, int QBUF, int NSTAGE>
 cudaError_t launch(dim3 grid, const CUtensorMap &mq, const CUtensorMap &mk, const CUtensorMap &mv,
-                   const vdx::AttnParams &p, cudaStream_t s)
+                   const vdx::AttnParams &p, const vdx::SegParams &sp, cudaStream_t s)
 {
-    vdx::attn_fwd_kernel<D, VARLEN, QBUF, NSTAGE>
-        <<<grid, vdx::NUM_THREADS, vdx::Layout<D, QBUF, NSTAGE>::ALLOC, s>>>(mq, mk, mv, p);
+    vdx::attn_fwd_kernel<D, MODE, QBUF, NSTAGE>
+        <<<grid, vdx::NUM_THREADS, vdx::Layout<D, QBUF, NSTAGE>::ALLOC, s>>>(mq, mk, mv, p, sp);
     return cudaGetLastError();
 }
 
@@ -119,7 +123,8 @@ int device_ready(int *sms = nullptr)
     return st.status;
 }
 
-// Workspace of the split tail, one per (device, stream): calls on one stream
+// Workspace of the split tail and of the segment key-tile lists, one per
+// (device, stream): calls on one stream
 // run in order, so they can share it; calls on different streams never do.
 // Allocated on the first call that needs it, grown when a later call needs
 // more (cudaFree waits for work still using the old one), kept until exit.
@@ -171,14 +176,26 @@ bool overlaps(const void *a, size_t na, const void *b, size_t nb)
     return x < y + nb && y < x + na;
 }
 
+// Per-problem-kind inputs: the valid key counts (MODE_VARLEN) or the
+// segment ids (MODE_SEG).
+struct KeyRule {
+    int mode = vdx::MODE_DENSE;
+    const int *kv_lens = nullptr;
+    const int *q_seg = nullptr;
+    const int *kv_seg = nullptr;
+};
+
 // fixed_scratch / fixed_bytes: when set, the split-tail workspace is taken
 // from that fixed device region instead of the library's allocation.
 int attn_launch(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
-                int D, const int *kv_lens, bool varlen, float scale, void *stream, void *fixed_scratch = nullptr,
+                int D, const KeyRule &rule, float scale, void *stream, void *fixed_scratch = nullptr,
                 size_t fixed_bytes = 0)
 {
+    const bool varlen = rule.mode == vdx::MODE_VARLEN;
+    const bool seg = rule.mode == vdx::MODE_SEG;
+    const int *kv_lens = rule.kv_lens;
     // ---- validation (no CUDA calls)
-    if (!q || !k || !v || !out || (varlen && !kv_lens))
+    if (!q || !k || !v || !out || (varlen && !kv_lens) || (seg && (!rule.q_seg || !rule.kv_seg)))
         return VDX_ERR_INVALID_ARG;
     if (B < 0 || H < 0 || Sq < 0 || Skv < 0)
         return VDX_ERR_INVALID_ARG;
@@ -187,7 +204,7 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     if (!std::isfinite(scale))
         return VDX_ERR_INVALID_ARG;
     if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(out, 16) || (lse && !aligned(lse, 4)) ||
-        (kv_lens && !aligned(kv_lens, 4)))
+        (kv_lens && !aligned(kv_lens, 4)) || (seg && (!aligned(rule.q_seg, 4) || !aligned(rule.kv_seg, 4))))
         return VDX_ERR_MISALIGNED;
     const long long bh = static_cast<long long>(B) * H;
     if (bh == 0 || Sq == 0)
@@ -217,6 +234,7 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         return st;
 
     vdx::AttnParams p{};
+    vdx::SegParams sp{};
     p.out = static_cast<__nv_bfloat16 *>(out);
     p.lse = lse;
     p.kv_lens = kv_lens;
@@ -248,7 +266,7 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     const int n_kv = (Skv + vdx::BN - 1) / vdx::BN;
     const int full_rounds = p.units / G;
     const int tail = p.units - full_rounds * G;
-    int parts = (!varlen && full_rounds >= 1 && tail > 0) ? G / tail : 0;
+    int parts = (rule.mode == vdx::MODE_DENSE && full_rounds >= 1 && tail > 0) ? G / tail : 0;
     if (parts > n_kv)
         parts = n_kv;
     if (parts >= 2) {
@@ -275,11 +293,52 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         if (cudaMemsetAsync(p.ws_count, 0, static_cast<size_t>(tail) * 4, s) != cudaSuccess)
             return VDX_ERR_CUDA;
     }
+    if (seg) {
+        // Key-tile lists per (sample, query-tile pair), shared by the heads.
+        const int n_qt = static_cast<int>(q_tiles);
+        const size_t pairs = static_cast<size_t>(B) * q_pairs;
+        const size_t kr_bytes = round_up(static_cast<size_t>(B) * n_kv * 8, 256);
+        const size_t qr_bytes = round_up(static_cast<size_t>(B) * n_qt * 8, 256);
+        const size_t list_bytes = round_up(pairs * n_kv * 4, 256);
+        const size_t cnt_bytes = round_up(pairs * 4, 256);
+        if (pairs * n_kv > static_cast<size_t>(INT_MAX))
+            return VDX_ERR_UNSUPPORTED;
+        int dev = 0;
+        void *ws = nullptr;
+        if (cudaGetDevice(&dev) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        if ((st = workspace(dev, s, kr_bytes + qr_bytes + list_bytes + cnt_bytes, &ws)) != VDX_OK)
+            return st;
+        char *base = static_cast<char *>(ws);
+        int2 *krange = reinterpret_cast<int2 *>(base);
+        int2 *qrange = reinterpret_cast<int2 *>(base + kr_bytes);
+        uint32_t *tlist = reinterpret_cast<uint32_t *>(base + kr_bytes + qr_bytes);
+        int *tcount = reinterpret_cast<int *>(base + kr_bytes + qr_bytes + list_bytes);
+        const long long range_warps = static_cast<long long>(B) * (n_kv + n_qt);
+        vdx::seg_tile_ranges_kernel<<<static_cast<unsigned>((range_warps + 7) / 8), 256, 0, s>>>(
+            rule.q_seg, rule.kv_seg, B, Sq, Skv, n_qt, n_kv, qrange, krange);
+        vdx::seg_tile_lists_kernel<<<static_cast<unsigned>((pairs + 7) / 8), 256, 0, s>>>(
+            qrange, krange, B, static_cast<int>(q_pairs), n_qt, n_kv, tlist, tcount);
+        if (cudaGetLastError() != cudaSuccess)
+            return VDX_ERR_CUDA;
+        sp.q_seg = rule.q_seg;
+        sp.kv_seg = rule.kv_seg;
+        sp.tlist = tlist;
+        sp.tcount = tcount;
+        sp.n_kt = n_kv;
+    }
+    using vdx::MODE_DENSE;
+    using vdx::MODE_SEG;
+    using vdx::MODE_VARLEN;
     cudaError_t e;
     if (D == 128) {
-        e = varlen ? launch<128, true, 1, 2>(grid, mq, mk, mv, p, s) : launch<128, false, 1, 2>(grid, mq, mk, mv, p, s);
+        e = varlen ? launch<128, MODE_VARLEN, 1, 2>(grid, mq, mk, mv, p, sp, s)
+                   : seg ? launch<128, MODE_SEG, 1, 2>(grid, mq, mk, mv, p, sp, s)
+                         : launch<128, MODE_DENSE, 1, 2>(grid, mq, mk, mv, p, sp, s);
     } else {
-        e = varlen ? launch<64, true, 2, 4>(grid, mq, mk, mv, p, s) : launch<64, false, 2, 4>(grid, mq, mk, mv, p, s);
+        e = varlen ? launch<64, MODE_VARLEN, 2, 4>(grid, mq, mk, mv, p, sp, s)
+                   : seg ? launch<64, MODE_SEG, 2, 4>(grid, mq, mk, mv, p, sp, s)
+                         : launch<64, MODE_DENSE, 2, 4>(grid, mq, mk, mv, p, sp, s);
     }
     if (e == cudaErrorNoKernelImageForDevice)
         return VDX_ERR_DEVICE;
@@ -338,12 +397,12 @@ int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out,
         !std::isfinite(scale))
         return VDX_ERR_INVALID_ARG;
     if (static_cast<long long>(B) * H == 0 || Sq == 0)
-        return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, nullptr, false, scale, stream);
+        return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, KeyRule{}, scale, stream);
     void *scratch = nullptr;
     const int st = noalloc_scratch(&scratch);
     if (st != VDX_OK)
         return st;
-    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, nullptr, false, scale, stream, scratch,
+    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, KeyRule{}, scale, stream, scratch,
                        kNoAllocScratchBytes);
 }
 
@@ -351,13 +410,26 @@ int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out,
 int vdx_attn_fwd(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
                  int D, float scale, void *stream)
 {
-    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, nullptr, false, scale, stream);
+    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, KeyRule{}, scale, stream);
 }
 
 int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,
                         int Skv_max, int D, const int *kv_lens, float scale, void *stream)
 {
-    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv_max, D, kv_lens, true, scale, stream);
+    KeyRule rule;
+    rule.mode = vdx::MODE_VARLEN;
+    rule.kv_lens = kv_lens;
+    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv_max, D, rule, scale, stream);
+}
+
+int vdx_attn_fwd_segments(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,
+                          int Skv, int D, const int *q_seg, const int *kv_seg, float scale, void *stream)
+{
+    KeyRule rule;
+    rule.mode = vdx::MODE_SEG;
+    rule.q_seg = q_seg;
+    rule.kv_seg = kv_seg;
+    return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, rule, scale, stream);
 }
 
 const char *vdx_status_string(int status)

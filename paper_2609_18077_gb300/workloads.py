@@ -75,11 +75,14 @@ class Workload:
     def segments(self) -> bool:
         return self.joint_text is not None
 
-    def flops(self, kv_lens=None) -> float:
+    def flops(self, kv_lens=None, q_seg=None, kv_seg=None) -> float:
         """Algorithmic FLOPs 4*B*H*Sq*Skv*D (two GEMMs, 2 flops per MAC).
 
-        With kv_lens the effective count uses the valid keys of each sample.
+        With kv_lens the effective count uses the valid keys of each sample;
+        with segment ids, the (query, key) pairs that share a segment.
         """
+        if q_seg is not None:
+            return 4.0 * self.H * self.D * float(segment_pairs(q_seg, kv_seg))
         if kv_lens is None:
             return 4.0 * self.B * self.H * self.Sq * self.Skv * self.D
         return 4.0 * self.H * self.Sq * self.D * float(np.sum(np.clip(kv_lens, 0, self.Skv)))
@@ -176,6 +179,17 @@ def joint_segments(text_lens, text_slots, S) -> np.ndarray:
     for b, L in enumerate(np.asarray(text_lens)):
         seg[b, int(L):text_slots] = 0
     return seg
+
+
+def segment_pairs(q_seg, kv_seg) -> int:
+    """Number of (query, key) pairs with equal segment ids, summed over samples."""
+    total = 0
+    for qs, ks in zip(np.asarray(q_seg), np.asarray(kv_seg)):
+        ids, qn = np.unique(qs, return_counts=True)
+        kid, kn = np.unique(ks, return_counts=True)
+        common, qi, ki = np.intersect1d(ids, kid, return_indices=True)
+        total += int(np.sum(qn[qi].astype(np.int64) * kn[ki].astype(np.int64)))
+    return total
 
 
 def pad_invalid_keys(k: torch.Tensor, v: torch.Tensor, kv_lens, fill_bits: int = BF16_NAN_BITS):

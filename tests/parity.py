@@ -54,9 +54,13 @@ def compare(o_gpu, lse_gpu, o_ref, lse_ref, rows=None):
     return max_abs, mean_abs, lse_rel
 
 
-def run_gpu(q, k, v, scale, kv_lens=None, device="cuda", with_lse=True):
+def run_gpu(q, k, v, scale, kv_lens=None, device="cuda", with_lse=True, q_seg=None, kv_seg=None):
     qd, kd, vd = (t.to(device) for t in (q, k, v))
-    if kv_lens is None:
+    if q_seg is not None:
+        qs = torch.from_numpy(np.ascontiguousarray(q_seg, dtype=np.int32)).to(device)
+        ks = torch.from_numpy(np.ascontiguousarray(kv_seg, dtype=np.int32)).to(device)
+        out, lse = binding.attn_fwd_segments(qd, kd, vd, qs, ks, scale=scale, return_lse=with_lse)
+    elif kv_lens is None:
         out, lse = binding.attn_fwd(qd, kd, vd, scale=scale, return_lse=with_lse)
     else:
         lens = torch.from_numpy(np.asarray(kv_lens, dtype=np.int32)).to(device)
@@ -66,15 +70,15 @@ def run_gpu(q, k, v, scale, kv_lens=None, device="cuda", with_lse=True):
     return out, lse
 
 
-def run_oracle(q, k, v, scale, kv_lens=None, rows=None):
+def run_oracle(q, k, v, scale, kv_lens=None, rows=None, q_seg=None, kv_seg=None):
     return oracle.attn_fwd(workloads.bf16_bits(q), workloads.bf16_bits(k), workloads.bf16_bits(v),
-                           scale, kv_lens=kv_lens, rows=rows)
+                           scale, kv_lens=kv_lens, rows=rows, q_seg=q_seg, kv_seg=kv_seg)
 
 
-def check_case(B, H, Sq, Skv, D, scale, seed, gain=1.0, kv_lens=None, rows=None):
+def check_case(B, H, Sq, Skv, D, scale, seed, gain=1.0, kv_lens=None, rows=None, q_seg=None, kv_seg=None):
     q, k, v = workloads.random_qkv(B, H, Sq, Skv, D, seed, gain)
     if kv_lens is not None:
         k, v = workloads.pad_invalid_keys(k, v, kv_lens)
-    out, lse = run_gpu(q, k, v, scale, kv_lens)
-    o_ref, lse_ref = run_oracle(q, k, v, scale, kv_lens, rows)
+    out, lse = run_gpu(q, k, v, scale, kv_lens, q_seg=q_seg, kv_seg=kv_seg)
+    o_ref, lse_ref = run_oracle(q, k, v, scale, kv_lens, rows, q_seg=q_seg, kv_seg=kv_seg)
     return compare(out, lse, o_ref, lse_ref, rows)

@@ -1,4 +1,4 @@
-"""Parity on the five video-shaped workloads at full size, in the bench's launch
+"""Parity on the video-shaped workloads at full size, in the bench's launch
 configuration, against the oracle on a seeded subset of query rows per head.
 
 The subset is the first VDX_PARITY_ROWS (default 1024) of the workload's
@@ -26,15 +26,16 @@ def _built():
     binding.load()
 
 
-@pytest.mark.parametrize("name", ["tiny", "small480", "cross", "large480", "large720"])
+@pytest.mark.parametrize("name", ["tiny", "small480", "cross", "large480", "large720", "joint45k"])
 def test_workload(name):
     from paper_2609_18077_gb300 import workloads
     w = workloads.generate(name)
     rows = w["rows"]
     if rows is not None:
         rows = np.ascontiguousarray(rows[:, :ROWS])
-    out, lse = run_gpu(w["q"], w["k"], w["v"], w["scale"], w["kv_lens"])
-    o_ref, lse_ref = run_oracle(w["q"], w["k"], w["v"], w["scale"], w["kv_lens"], rows)
+    out, lse = run_gpu(w["q"], w["k"], w["v"], w["scale"], w["kv_lens"], q_seg=w["q_seg"], kv_seg=w["kv_seg"])
+    o_ref, lse_ref = run_oracle(w["q"], w["k"], w["v"], w["scale"], w["kv_lens"], rows, q_seg=w["q_seg"],
+                                kv_seg=w["kv_seg"])
     stats = compare(out, lse, o_ref, lse_ref, rows)
     print(f"{name}: O max {stats[0]:.3e} mean {stats[1]:.3e} LSE rel {stats[2]:.3e}")
     del out, lse

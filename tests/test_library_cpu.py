@@ -70,6 +70,19 @@ def test_varlen_requires_lengths(lib):
                                    0.1, None) == 3
 
 
+def test_segments_require_ids(lib):
+    g = GOOD
+    args = (g["q"], g["k"], g["v"], g["out"], g["lse"], 1, 1, 8, 8, 128)
+    assert lib.vdx_attn_fwd_segments(*args, None, 7 * A, 0.1, None) == 1
+    assert lib.vdx_attn_fwd_segments(*args, 6 * A, None, 0.1, None) == 1
+    assert lib.vdx_attn_fwd_segments(*args, 6 * A + 2, 7 * A, 0.1, None) == 3
+    assert lib.vdx_attn_fwd_segments(*args, 6 * A, 7 * A + 1, 0.1, None) == 3
+    assert lib.vdx_attn_fwd_segments(g["q"], g["k"], g["v"], g["out"], g["lse"], 1, 1, 8, 8, 80,
+                                     6 * A, 7 * A, 0.1, None) == 1
+    assert lib.vdx_attn_fwd_segments(g["q"], g["k"], g["v"], g["out"], g["lse"], 0, 1, 8, 8, 128,
+                                     6 * A, 7 * A, 0.1, None) == 0
+
+
 def test_selftest_limit_validation(lib):
     assert lib.vdx_selftest_wait_timeout(0, None) == 1
     assert lib.vdx_selftest_wait_timeout(10000001, None) == 1
