@@ -143,9 +143,10 @@ struct Layout {
     static constexpr int TMEM_PTR_OFF = BAR_OFF + NBARS * 8;
     static constexpr int ABORT_OFF = TMEM_PTR_OFF + 4;
     static constexpr int MERGE_OFF = ABORT_OFF + 4;          // "this CTA merges" flag
+    static constexpr int ENTRY_OFF = MERGE_OFF + 4;          // [NSTAGE] MODE_SEG: list entry of each stage's V tile
     // 197.8 KB in all configurations: under the 196 KB shared-memory carve-out
     // (199,680 usable bytes), which leaves 60 KB of L1 for the spill slots.
-    static constexpr int BYTES = MERGE_OFF + 4;
+    static constexpr int BYTES = ENTRY_OFF + 4 * NSTAGE;
     static constexpr int ALLOC = BYTES + 1024;               // slack for 1024-B alignment
 };
 
@@ -445,13 +446,14 @@ __device__ __forceinline__ Item item_at(const AttnParams &p, const SegParams &sp
     return w;
 }
 
-// Key tile of list position r of item w (the identity unless MODE_SEG).
+// List entry of position r of item w: in MODE_SEG the key tile and its mask
+// bits (segment_tiles.cuh); otherwise the key tile r itself.
 template <int MODE>
-__device__ __forceinline__ int key_tile(const SegParams &sp, const Item &w, int r)
+__device__ __forceinline__ uint32_t tile_entry(const SegParams &sp, const Item &w, int r)
 {
     if (MODE == MODE_SEG)
-        return static_cast<int>(__ldg(sp.tlist + w.list_off + r) & SEG_TILE_BITS);
-    return r;
+        return __ldg(sp.tlist + w.list_off + r);
+    return static_cast<uint32_t>(r);
 }
 
 template <int D, int MODE, int QBUF, int NSTAGE>
@@ -526,8 +528,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         int g = 0;
         int fixes = 0;
         bool ok = true;
-        // load stage g: V tile (vbh, vj) if vj >= 0, K tile (kbh, kj) if kj >= 0
-        auto stage = [&](int vbh, int vj, int v_valid, int kbh, int kj) -> bool {
+        // load stage g: V tile (vbh, vj) if vj >= 0, K tile (kbh, kj) if kj >= 0.
+        // MODE_SEG: the V tile's list entry goes to the stage's slot before the
+        // full barrier is armed (its arrive releases the slot to the softmax,
+        // which reads it after its wait on that barrier; the slot is rewritten
+        // only after the stage is released, i.e. after that read).
+        auto stage = [&](int vbh, int vj, int v_valid, int kbh, int kj, uint32_t ventry) -> bool {
             const int st = g % L::NSTAGE;
             const int rnd = g / L::NSTAGE;
             ++g;
@@ -563,6 +569,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             if (lane == 0) {
                 const uint32_t bytes = ((has_v && !fix) + has_k) * L::TILE_BYTES;
+                if (MODE == MODE_SEG && has_v)
+                    reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF)[st] = ventry;
                 if (bytes) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_FULL + st), bytes);
                     for (int h = 0; h < D / 64; ++h) {
@@ -589,7 +597,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         if (i >= 0) {
             const Item w = item_at<MODE>(p, sp, cta, i);
-            ok = stage(0, -1, BN, w.bh, key_tile<MODE>(sp, w, w.j0));
+            ok = stage(0, -1, BN, w.bh, static_cast<int>(tile_entry<MODE>(sp, w, w.j0) & SEG_TILE_BITS), 0u);
         }
         for (int iq = 0; ok && i >= 0; ++iq) {
             const Item w = item_at<MODE>(p, sp, cta, i);
@@ -615,14 +623,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             nw.ok = false;
             if (ni >= 0)
                 nw = item_at<MODE>(p, sp, cta, ni);
-            int vj = key_tile<MODE>(sp, w, w.j0);
+            uint32_t ve = tile_entry<MODE>(sp, w, w.j0);
             for (int j = w.j0; ok && j < w.j1; ++j) {
                 const bool last = j + 1 == w.j1;
                 const int kbh = last ? (nw.ok ? nw.bh : 0) : w.bh;
                 // MODE_SEG: the list entry is read before the stage's empty wait
-                const int kj = last ? (nw.ok ? key_tile<MODE>(sp, nw, nw.j0) : -1) : key_tile<MODE>(sp, w, j + 1);
-                ok = stage(w.bh, vj, w.kv_valid - vj * BN, kbh, kj);
-                vj = kj;
+                const uint32_t ke = last ? (nw.ok ? tile_entry<MODE>(sp, nw, nw.j0) : 0u) : tile_entry<MODE>(sp, w, j + 1);
+                const int kj = (last && !nw.ok) ? -1 : static_cast<int>(ke & SEG_TILE_BITS);
+                const int vj = static_cast<int>(ve & SEG_TILE_BITS);
+                ok = stage(w.bh, vj, w.kv_valid - vj * BN, kbh, kj, ve);
+                ve = ke;
             }
             i = ni;
         }
@@ -753,45 +763,17 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             float m_used = -INFINITY;
             float l_exact = 0.f;   // sum of the fp32 weights: the log-sum-exp
             float l_resid = 0.f;   // sum over tiles of r - p for each tile's largest weight
-            // MODE_SEG: this row's segment id, the sample's key ids and the next list entry
-            int my_seg = 0;
-            const int *kseg = nullptr;
-            uint32_t next_entry = 0;
-            if (MODE == MODE_SEG) {
-                const size_t b = static_cast<size_t>(w.bh / p.H);
-                my_seg = store ? __ldg(sp.q_seg + b * p.Sq + q_row) : 0;
-                kseg = sp.kv_seg + b * p.Skv;
-                next_entry = __ldg(sp.tlist + w.list_off + w.j0);
-            }
             for (int j = w.j0; j < w.j1; ++j, ++sc) {
-                int kt = j;   // key tile
-                bool seg_mask = false;
-                int ids[4];
-                if (MODE == MODE_SEG) {
-                    const uint32_t entry = next_entry;
-                    kt = static_cast<int>(entry & SEG_TILE_BITS);
-                    if (j + 1 < w.j1)
-                        next_entry = __ldg(sp.tlist + w.list_off + j + 1);
-                    seg_mask = (entry >> (SEG_MASK_SHIFT + t)) & 1u;
-                    if (seg_mask) {
-                        // this lane's four of the tile's 128 key ids, read under the S wait
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const int c = kt * BN + e * 32 + lane;
-                            ids[e] = c < p.Skv ? __ldg(kseg + c) : 0;
-                        }
-                    }
-                }
                 if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_S + t), sc & 1, abort_flag, limit))))
                     break;
                 ptx::tc_fence_after_sync();
+                const int gj = g + (j - w.j0);
                 uint32_t s[4][32];
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
                     ptx::tmem_ld32(s_addr + 32 * c, s[c]);
                 // The stage (V_j, next K) must have landed before P_t(j) is
                 // published; checked here, under the TMEM load latency.
-                const int gj = g + (j - w.j0);
                 if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + gj % L::NSTAGE),
                                                                 (gj / L::NSTAGE) & 1, abort_flag, limit)))) {
                     ptx::tmem_wait_ld();
@@ -799,6 +781,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 ptx::tmem_wait_ld();
 
+                int kt = j;   // key tile
+                bool seg_mask = false;
+                if (MODE == MODE_SEG) {
+                    // the stage's list entry, published with its full barrier
+                    const uint32_t entry = reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF)[gj % L::NSTAGE];
+                    kt = static_cast<int>(entry & SEG_TILE_BITS);
+                    seg_mask = (entry >> (SEG_MASK_SHIFT + t)) & 1u;
+                }
                 const int valid = w.kv_valid - kt * BN;
                 if (valid < BN) {
                     // Ragged last tile: keys past the end (or past the sample's
@@ -812,9 +802,19 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 if (MODE == MODE_SEG && seg_mask) {
                     // Keys of another segment get the masked logit too.  Lane
-                    // l holds the ids of keys 32e + l; the warp shares them by
-                    // shuffles (a marked tile is rare: segment borders only).
+                    // l reads the ids of keys 32e + l and the warp shares them by
+                    // shuffles (a marked tile is rare: segment borders only, so
+                    // the load latency is taken here rather than kept in flight).
                     const uint32_t pad = neg_scale ? 0x7F800000u : 0xFF800000u;
+                    const size_t b = static_cast<size_t>(w.bh / p.H);
+                    const int my_seg = store ? __ldg(sp.q_seg + b * p.Sq + q_row) : 0;
+                    const int *kseg = sp.kv_seg + b * p.Skv;
+                    int ids[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int c = kt * BN + e * 32 + lane;
+                        ids[e] = c < p.Skv ? __ldg(kseg + c) : 0;
+                    }
 #pragma unroll
                     for (int c = 0; c < BN; ++c) {
                         const int kid = __shfl_sync(0xffffffffu, ids[c >> 5], c & 31);
