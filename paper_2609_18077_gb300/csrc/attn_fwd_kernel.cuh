@@ -938,6 +938,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             g += w.j1 - w.j0;
             ++iq;
         }
+        // An abort can leave this warp's tensor-memory loads or stores in
+        // flight; none may remain when the memory is released below.
+        ptx::tmem_wait_ld();
+        ptx::tmem_wait_st();
     }
 
     ptx::tc_fence_before_sync();
