@@ -56,6 +56,11 @@ class Oracle:
             ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
             ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
             ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
+        lib.oracle_rope3d.restype = ctypes.c_int
+        lib.oracle_rope3d.argtypes = [
+            ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_double, ctypes.c_int, ctypes.c_void_p]
         lib.oracle_set_threads.restype = ctypes.c_int
         lib.oracle_set_threads.argtypes = [ctypes.c_int]
         self._lib = lib
@@ -119,6 +124,24 @@ class Oracle:
         return (o, lse, pr) if probs else (o, lse)
 
 
+    def rope3d(self, x, grid, s0, dims, theta, interleaved=True):
+        """3D rotary embedding in fp64 (see oracle.c).
+
+        x: uint16 [B,H,S,D] bf16 bits; grid = (F, Hp, Wp); tokens [s0, s0+F*Hp*Wp)
+        are the video grid; dims = (d_t, d_h, d_w).  Returns float64 [B,H,S,D].
+        """
+        x = _bits(x)
+        B, H, S, D = x.shape
+        F, Hp, Wp = grid
+        y = np.empty((B, H, S, D), dtype=np.float64)
+        rc = self._lib.oracle_rope3d(_ptr(x), B, H, S, D, int(F), int(Hp), int(Wp), int(s0),
+                                     int(dims[0]), int(dims[1]), int(dims[2]), float(theta), int(bool(interleaved)),
+                                     _ptr(y))
+        if rc != 0:
+            raise RuntimeError("oracle_rope3d rejected its arguments")
+        return y
+
+
 def _bits(a) -> np.ndarray:
     a = np.asarray(a)
     if a.dtype != np.uint16 or a.ndim != 4:
@@ -141,6 +164,11 @@ def default() -> Oracle:
             build()
         _default = Oracle(LIBRARY)
     return _default
+
+
+def rope3d(x, grid, s0, dims, theta, interleaved=True):
+    """Module-level shortcut for ``default().rope3d``."""
+    return default().rope3d(x, grid, s0, dims, theta, interleaved)
 
 
 def attn_fwd(q, k, v, scale, kv_lens=None, rows=None, probs=False, q_seg=None, kv_seg=None):

@@ -33,6 +33,19 @@
  * the definition above runs over that key set in ascending key order.  A query
  * whose segment owns no key gets o = 0 and lse = -inf.
  *
+ * 3D rotary position embedding (oracle_rope3d).  Sec. 2 of the paper
+ * ("3D RoPE, 3D VAEs, and flash attention") keeps each model family's own
+ * 3D RoPE convention over time, height and width without stating one.  The
+ * oracle is the standard rotary embedding over a 3-D grid, parameterised by
+ * the conventions those families differ in: the video tokens [s0, s0 + F*Hp*Wp)
+ * of a sequence sit at grid positions (t, h, w) in raster order; the first
+ * d_t head dims rotate with t, the next d_h with h, the next d_w with w, the
+ * rest are untouched; inside an axis part of d_a dims, pair i is (2i, 2i+1)
+ * (interleaved) or (i, i + d_a/2) (half split) and turns by the angle
+ * pos * theta^(-2i/d_a):
+ *     (y_a, y_b) = (x_a cos(phi) - x_b sin(phi), x_a sin(phi) + x_b cos(phi)).
+ * Tokens outside the grid are copied unchanged.  Output is fp64.
+ *
  * Inputs are bf16 bit patterns (uint16), decoded exactly to fp64.  All
  * arithmetic is fp64.  Layout: q [B,H,Sq,D], k and v [B,H,Skv,D], contiguous.
  * Parallelism: one OpenMP loop over (b, h, query row); each row is computed
@@ -245,6 +258,48 @@ int oracle_attn_fwd_seg(const uint16_t *q, const uint16_t *k, const uint16_t *v,
         free(idx);
     }
     return failed ? -1 : 0;
+}
+
+/*
+ * 3D rotary embedding of x [B, H, S, D] (bf16 bits) into y (fp64, same shape);
+ * see the header for the parameters.  Returns 0, or -1 on a bad argument.
+ */
+int oracle_rope3d(const uint16_t *x, int B, int H, int S, int D, int F, int Hp, int Wp, int s0,
+                  int d_t, int d_h, int d_w, double theta, int interleaved, double *y)
+{
+    if (!x || !y || B < 0 || H < 0 || S < 0 || D <= 0 || F < 0 || Hp < 0 || Wp < 0 || s0 < 0 ||
+        d_t < 0 || d_h < 0 || d_w < 0 || (d_t | d_h | d_w) & 1 || d_t + d_h + d_w > D || !(theta > 0.0))
+        return -1;
+    const long rows = (long)B * H * S;
+    const long grid = (long)F * Hp * Wp;
+#pragma omp parallel for schedule(static)
+    for (long r = 0; r < rows; ++r) {
+        const long s = r % S;
+        const uint16_t *xr = x + (size_t)r * D;
+        double *yr = y + (size_t)r * D;
+        for (int d = 0; d < D; ++d)
+            yr[d] = bf16_to_f64(xr[d]);
+        const long g = s - s0;
+        if (g < 0 || g >= grid)
+            continue;
+        /* grid position of this token, raster order (t, h, w) */
+        const long pos[3] = {g / ((long)Hp * Wp), (g / Wp) % Hp, g % Wp};
+        const int len[3] = {d_t, d_h, d_w};
+        int base = 0;
+        for (int a = 0; a < 3; ++a) {
+            const int da = len[a];
+            for (int i = 0; i < da / 2; ++i) {
+                const double phi = (double)pos[a] * pow(theta, -2.0 * i / da);
+                const int ia = base + (interleaved ? 2 * i : i);
+                const int ib = base + (interleaved ? 2 * i + 1 : i + da / 2);
+                const double xa = bf16_to_f64(xr[ia]), xb = bf16_to_f64(xr[ib]);
+                yr[ia] = xa * cos(phi) - xb * sin(phi);
+                yr[ib] = xa * sin(phi) + xb * cos(phi);
+            }
+            base += da;
+        }
+    }
+    return 0;
 }
 
 /* Threads the OpenMP loop may use (n <= 0 keeps the runtime default). */

@@ -19,6 +19,10 @@ Sources of the facts (none of them is the oracle's own code):
     segment everywhere is dense attention; packed segments are independent
     problems; a prefix segment is the valid-count form; torch's SDPA with the
     boolean mask q_seg[i] == kv_seg[j];
+  * 3D RoPE: the textbook complex form z exp(i phi), norm preservation,
+    identity off the grid and at its origin, one axis per coordinate, dot
+    products depending on relative position only, and the two pairings
+    agreeing up to a permutation of dims;
   * torch's scaled_dot_product_attention and logsumexp in fp64 (a library);
   * a 50-digit mpmath evaluation on a tiny input.
 """
@@ -303,9 +307,114 @@ def pin_segments_torch_masked_sdpa(orc):
     np.testing.assert_allclose(p.sum(-1)[has], 1.0, rtol=0, atol=1e-13)
 
 
+# ---- 3D rotary position embedding (Sec. 2: each family keeps its own 3D RoPE convention)
+
+def _rope_x(B, H, S, D, seed, gain=1.0):
+    q, _, _ = random_qkv(B, H, S, 1, D, seed, gain)
+    return bf16_bits(q)
+
+
+def pin_rope_complex_rotation(orc):
+    """Each pair, read as a complex number z = x_a + i x_b, becomes z * exp(i phi)
+    with phi = pos * theta^(-2i/d_a) (the textbook complex form, numpy complex exp)."""
+    F, Hp, Wp, s0, D = 2, 3, 4, 2, 32
+    dims, theta = (8, 12, 10), 100.0
+    S = s0 + F * Hp * Wp + 3
+    x = _rope_x(1, 2, S, D, seed=31)
+    xd = _dec(x)
+    for inter in (True, False):
+        y = orc.rope3d(x, (F, Hp, Wp), s0, dims, theta, inter)
+        for s in range(s0, s0 + F * Hp * Wp):
+            g = s - s0
+            pos = (g // (Hp * Wp), (g // Wp) % Hp, g % Wp)
+            base = 0
+            for a, da in enumerate(dims):
+                for i in range(da // 2):
+                    ia, ib = (base + 2 * i, base + 2 * i + 1) if inter else (base + i, base + i + da // 2)
+                    z = (xd[:, :, s, ia] + 1j * xd[:, :, s, ib]) * np.exp(1j * pos[a] * theta ** (-2.0 * i / da))
+                    np.testing.assert_allclose(y[:, :, s, ia], z.real, rtol=0, atol=1e-12)
+                    np.testing.assert_allclose(y[:, :, s, ib], z.imag, rtol=0, atol=1e-12)
+                base += da
+
+
+def pin_rope_norm_and_identity(orc):
+    """Rotations keep every pair's norm; the grid origin, tokens outside the grid and
+    the dims past d_t + d_h + d_w are unchanged."""
+    F, Hp, Wp, s0, D = 3, 2, 5, 4, 40
+    dims = (10, 8, 12)
+    S = s0 + F * Hp * Wp + 6
+    x = _rope_x(2, 1, S, D, seed=32, gain=2.0)
+    xd = _dec(x)
+    y = orc.rope3d(x, (F, Hp, Wp), s0, dims, 10000.0, True)
+    np.testing.assert_allclose(np.sum(y[..., :30].reshape(2, 1, S, 15, 2) ** 2, -1),
+                               np.sum(xd[..., :30].reshape(2, 1, S, 15, 2) ** 2, -1), rtol=1e-13, atol=1e-13)
+    np.testing.assert_array_equal(y[..., 30:], xd[..., 30:])
+    outside = list(range(s0)) + list(range(s0 + F * Hp * Wp, S))
+    np.testing.assert_array_equal(y[:, :, outside], xd[:, :, outside])
+    np.testing.assert_array_equal(y[:, :, s0], xd[:, :, s0])          # position (0, 0, 0)
+
+
+def pin_rope_one_axis_each(orc):
+    """A step along t turns only the t dims, along h only the h dims, along w only the w dims."""
+    F, Hp, Wp, D = 2, 2, 2, 24
+    dims = (8, 8, 8)
+    x = _rope_x(1, 1, F * Hp * Wp, D, seed=33)
+    xd = _dec(x)
+    y = orc.rope3d(x, (F, Hp, Wp), 0, dims, 50.0, False)
+    for s, axis in ((4, 0), (2, 1), (1, 2)):          # (1,0,0), (0,1,0), (0,0,1)
+        for a in range(3):
+            sl = slice(8 * a, 8 * a + 8)
+            if a == axis:
+                assert np.max(np.abs(y[0, 0, s, sl] - xd[0, 0, s, sl])) > 1e-3
+            else:
+                np.testing.assert_array_equal(y[0, 0, s, sl], xd[0, 0, s, sl])
+
+
+def pin_rope_relative_position(orc):
+    """<R(p) q, R(p') k> depends on p - p' only: moving both tokens by the same step
+    along any axis leaves their dot product unchanged."""
+    F, Hp, Wp, D = 4, 4, 4, 48
+    dims = (16, 16, 16)
+    S = F * Hp * Wp
+    rng = np.random.default_rng(34)
+    qv = _bits_of(rng.standard_normal(D).astype(np.float32))
+    kv = _bits_of(rng.standard_normal(D).astype(np.float32))
+    idx = lambda t, h, w: (t * Hp + h) * Wp + w
+    x = np.zeros((1, 1, S, D), dtype=np.uint16)
+    pairs = [((0, 1, 2), (1, 0, 0)), ((1, 2, 3), (2, 1, 1))]   # second pair = first shifted by (1, 1, 1)
+    for (pq, pk) in pairs:
+        x[0, 0, idx(*pq)] = qv
+        x[0, 0, idx(*pk)] = kv
+    for inter in (True, False):
+        y = orc.rope3d(x, (F, Hp, Wp), 0, dims, 1000.0, inter)
+        d0 = y[0, 0, idx(*pairs[0][0])] @ y[0, 0, idx(*pairs[0][1])]
+        d1 = y[0, 0, idx(*pairs[1][0])] @ y[0, 0, idx(*pairs[1][1])]
+        assert abs(d0 - d1) <= 1e-11 * max(1.0, abs(d0)), (d0, d1)
+
+
+def pin_rope_pairing_conventions(orc):
+    """The half-split pairing is the interleaved one on dims permuted inside each axis
+    part (interleaved 2i, 2i+1 <-> half i, i + d_a/2)."""
+    F, Hp, Wp, D = 2, 3, 2, 30
+    dims = (6, 10, 12)
+    x = _rope_x(1, 2, F * Hp * Wp, D, seed=35)
+    perm = np.arange(D)
+    base = 0
+    for da in dims:
+        for i in range(da // 2):
+            perm[base + 2 * i] = base + i
+            perm[base + 2 * i + 1] = base + i + da // 2
+        base += da
+    yi = orc.rope3d(np.ascontiguousarray(x[..., perm]), (F, Hp, Wp), 0, dims, 77.0, True)
+    yh = orc.rope3d(x, (F, Hp, Wp), 0, dims, 77.0, False)
+    np.testing.assert_allclose(yi, yh[..., perm], rtol=0, atol=1e-13)
+
+
 ALL_PINS = [pin_single_key, pin_two_keys, pin_weights_sum_to_one, pin_constant_values,
             pin_zero_logits, pin_query_permutation, pin_key_value_permutation,
             pin_value_translation, pin_varlen_is_truncation, pin_varlen_empty_and_clamped,
             pin_row_subset, pin_torch_sdpa, pin_mpmath_brute_force, pin_large_logits_stable,
             pin_segments_one_segment_is_dense, pin_segments_packed_are_independent,
-            pin_segments_prefix_is_valid_count, pin_segments_torch_masked_sdpa]
+            pin_segments_prefix_is_valid_count, pin_segments_torch_masked_sdpa,
+            pin_rope_complex_rotation, pin_rope_norm_and_identity, pin_rope_one_axis_each,
+            pin_rope_relative_position, pin_rope_pairing_conventions]

@@ -43,6 +43,16 @@ MUTANTS = {
     "seg_k_by_position": [("const size_t kj = (size_t)(idx ? idx[j] : j);", "const size_t kj = (size_t)j;")],
     "seg_v_by_position": [("const size_t vj = (size_t)(idx ? idx[j] : j);", "const size_t vj = (size_t)j;")],
     "seg_probs_by_position": [("pr[idx[e]] = ps[e];", "pr[e] = ps[e];")],
+    "rope_sign": [("yr[ia] = xa * cos(phi) - xb * sin(phi);", "yr[ia] = xa * cos(phi) + xb * sin(phi);")],
+    "rope_direction": [("yr[ia] = xa * cos(phi) - xb * sin(phi);", "yr[ia] = xa * cos(phi) + xb * sin(phi);"),
+                       ("yr[ib] = xa * sin(phi) + xb * cos(phi);", "yr[ib] = -xa * sin(phi) + xb * cos(phi);")],
+    "rope_freq_exponent": [("pow(theta, -2.0 * i / da)", "pow(theta, -1.0 * i / da)")],
+    "rope_raster_h": [("(g / Wp) % Hp", "g % Hp")],
+    "rope_t_from_w": [("g / ((long)Hp * Wp)", "g / Wp")],
+    "rope_pairs_swapped": [("(interleaved ? 2 * i : i)", "(interleaved ? i : 2 * i)"),
+                           ("(interleaved ? 2 * i + 1 : i + da / 2)", "(interleaved ? i + da / 2 : 2 * i + 1)")],
+    "rope_base_fixed": [("            base += da;\n        }\n    }\n    return 0;", "        }\n    }\n    return 0;")],
+    "rope_offset_ignored": [("const long g = s - s0;", "const long g = s;")],
 }
 
 CHILD = r"""
