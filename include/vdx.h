@@ -108,6 +108,26 @@ int vdx_attn_fwd_segments(const void *q, const void *k, const void *v, void *out
                           float scale, void *stream);
 
 /*
+ * 3D rotary position embedding of queries or keys (Sec. 2: each model family
+ * keeps its own 3D RoPE convention over time, height and width; this call
+ * takes the conventions as parameters).  The standard rotary embedding over a
+ * token grid:
+ *   x, y : bf16 [B, H, S, D], DEVICE pointers, caller-owned, 4-byte aligned;
+ *          y == x rotates in place, otherwise the two must not overlap.
+ *   F, Hp, Wp, s0 : tokens [s0, s0 + F*Hp*Wp) of each sequence are the video
+ *          grid, in raster order (t, h, w); other tokens are copied unchanged.
+ *   d_t, d_h, d_w : even numbers of head dims turned by t, h and w, taken in
+ *          that order from dim 0; d_t + d_h + d_w <= D; the rest are copied.
+ *   theta : frequency base (> 0).  Pair i of an axis part of d_a dims turns by
+ *          pos * theta^(-2i/d_a):  (y_a, y_b) = (x_a cos - x_b sin, x_a sin + x_b cos).
+ *   interleaved : 1: pairs (2i, 2i+1) of the part; 0: pairs (i, i + d_a/2).
+ * D must be even, 2 .. 512.  Arithmetic in fp32, y rounded to bf16 (nearest
+ * even).  Asynchronous on `stream`; allocates nothing.
+ */
+int vdx_rope3d(const void *x, void *y, int B, int H, int S, int D, int F, int Hp, int Wp, int s0,
+               int d_t, int d_h, int d_w, float theta, int interleaved, void *stream);
+
+/*
  * vdx_attn_fwd without any device allocation (the paper has no counterpart;
  * this is a library service).  Same arguments, results and errors as
  * vdx_attn_fwd, for callers that must not allocate device memory: code that

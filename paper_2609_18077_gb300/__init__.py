@@ -5,4 +5,4 @@ The compute path is the CUDA library ``_lib/libvdx.so`` (C ABI in
 it.  The library is loaded on first use and its absence is an error.
 """
 from .binding import (VdxError, attn_fwd, attn_fwd_segments, attn_fwd_varlen, check_device_error, load,  # noqa: F401
-                      selftest_wait_timeout, status_string, version)
+                      rope3d, selftest_wait_timeout, status_string, version)

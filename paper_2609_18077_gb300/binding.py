@@ -33,6 +33,7 @@ SIGNATURES = {
     "vdx_attn_fwd_varlen": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, ctypes.c_float, _P]),
     "vdx_attn_fwd_segments": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, ctypes.c_float, _P]),
     "vdx_attn_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, ctypes.c_float, _P]),
+    "vdx_rope3d": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _I, _I, _I, ctypes.c_float, _I, _P]),
     "vdx_status_string": (ctypes.c_char_p, [_I]),
     "vdx_check_device_error": (_I, [_P]),
     "vdx_selftest_wait_timeout": (_I, [_I, _P]),
@@ -182,3 +183,28 @@ def attn_fwd_segments(q, k, v, q_seg, kv_seg, scale=None, out=None, lse=None, re
     if st != VDX_OK:
         raise VdxError(st, "vdx_attn_fwd_segments")
     return out, lse
+
+
+def rope3d(x, grid, s0, dims, theta, interleaved=True, out=None):
+    """3D rotary position embedding through ``vdx_rope3d``.
+
+    x: bf16 CUDA tensor [B,H,S,D]; grid = (F, Hp, Wp): tokens [s0, s0 + F*Hp*Wp)
+    are the video grid in raster order; dims = (d_t, d_h, d_w).  out=x rotates
+    in place; out=None allocates the result.  Returns out.
+    """
+    if not isinstance(x, torch.Tensor) or not x.is_cuda or x.dtype != torch.bfloat16 or x.dim() != 4 \
+            or not x.is_contiguous():
+        raise TypeError("x must be a contiguous bf16 CUDA tensor [B,H,S,D]")
+    if out is None:
+        out = torch.empty_like(x)
+    elif out.shape != x.shape or out.dtype != x.dtype or not out.is_contiguous() or out.device != x.device:
+        raise ValueError("out must be a contiguous bf16 tensor shaped like x on x's device")
+    B, H, S, D = x.shape
+    F, Hp, Wp = (int(v) for v in grid)
+    d_t, d_h, d_w = (int(v) for v in dims)
+    with torch.cuda.device(x.device):
+        st = load().vdx_rope3d(x.data_ptr(), out.data_ptr(), B, H, S, D, F, Hp, Wp, int(s0), d_t, d_h, d_w,
+                               float(theta), int(bool(interleaved)), _stream_handle(x.device))
+    if st != VDX_OK:
+        raise VdxError(st, "vdx_rope3d")
+    return out

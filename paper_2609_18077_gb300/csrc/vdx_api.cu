@@ -18,6 +18,7 @@
 #include <utility>
 
 #include "attn_fwd_kernel.cuh"
+#include "rope3d.cuh"
 #include "vdx.h"
 
 namespace {
@@ -420,6 +421,69 @@ int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, 
     rule.mode = vdx::MODE_VARLEN;
     rule.kv_lens = kv_lens;
     return attn_launch(q, k, v, out, lse, B, H, Sq, Skv_max, D, rule, scale, stream);
+}
+
+int vdx_rope3d(const void *x, void *y, int B, int H, int S, int D, int F, int Hp, int Wp, int s0, int d_t, int d_h,
+               int d_w, float theta, int interleaved, void *stream)
+{
+    // ---- validation (no CUDA calls)
+    if (!x || !y || B < 0 || H < 0 || S < 0 || F < 0 || Hp < 0 || Wp < 0 || s0 < 0)
+        return VDX_ERR_INVALID_ARG;
+    if (D < 2 || D > 512 || (D & 1) || d_t < 0 || d_h < 0 || d_w < 0 || ((d_t | d_h | d_w) & 1) ||
+        static_cast<long long>(d_t) + d_h + d_w > D)
+        return VDX_ERR_INVALID_ARG;
+    if (!std::isfinite(theta) || !(theta > 0.f))
+        return VDX_ERR_INVALID_ARG;
+    if (!aligned(x, 4) || !aligned(y, 4))
+        return VDX_ERR_MISALIGNED;
+    const long long bh = static_cast<long long>(B) * H;
+    if (bh == 0 || S == 0)
+        return VDX_OK;
+    if (bh > INT_MAX)
+        return VDX_ERR_INVALID_ARG;
+    const size_t bytes = static_cast<size_t>(bh) * S * D * 2;
+    if (x != y && overlaps(x, bytes, y, bytes))
+        return VDX_ERR_INVALID_ARG;
+    // ---- device set-up and launch
+    int sms = 0;
+    const int st = device_ready(&sms);
+    if (st != VDX_OK)
+        return st;
+    vdx::RopeParams p{};
+    p.x = static_cast<const __nv_bfloat16 *>(x);
+    p.y = static_cast<__nv_bfloat16 *>(y);
+    p.BH = static_cast<int>(bh);
+    p.S = S;
+    p.D = D;
+    p.F = F;
+    p.Hp = Hp;
+    p.Wp = Wp;
+    p.s0 = s0;
+    p.d_t = d_t;
+    p.d_h = d_h;
+    p.d_w = d_w;
+    p.log2_theta = static_cast<float>(std::log2(static_cast<double>(theta)));
+    p.copy_all = x != y;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (interleaved && D % 8 == 0 && aligned(x, 16) && aligned(y, 16)) {
+        // 16-byte chunks: four pairs per thread
+        const int chunks = D / 8;
+        const int tok = 256 / chunks;
+        const long long groups = (S + tok - 1) / tok;
+        const long long cap = static_cast<long long>(sms) * vdx::ROPE_VEC_BLOCKS_PER_SM;
+        const unsigned nb = static_cast<unsigned>(groups < cap ? groups : cap);
+        vdx::rope3d_vec_kernel<<<dim3(nb), dim3(static_cast<unsigned>(chunks), static_cast<unsigned>(tok)), 0, s>>>(p);
+    } else {
+        const int pairs = D / 2;
+        const int tok = 256 / pairs;
+        const dim3 block(static_cast<unsigned>(pairs), static_cast<unsigned>(tok));
+        const dim3 grid(static_cast<unsigned>((S + tok - 1) / tok));
+        if (interleaved)
+            vdx::rope3d_kernel<true><<<grid, block, 0, s>>>(p);
+        else
+            vdx::rope3d_kernel<false><<<grid, block, 0, s>>>(p);
+    }
+    return cudaGetLastError() == cudaSuccess ? VDX_OK : VDX_ERR_CUDA;
 }
 
 int vdx_attn_fwd_segments(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,

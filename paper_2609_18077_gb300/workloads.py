@@ -24,6 +24,10 @@ Recipe (every draw is seeded; no dataset is read):
     [lo, hi]; K/V rows past a sample's length are padding and may be filled
     with NaN to prove they are never read;
   * row subsets for large configs: per (b, h), n distinct query rows;
+  * 3D RoPE (Sec. 2: each family keeps its own convention): the rope480
+    workload rotates small480's Q and K over its 21x30x52 grid with Wan's
+    published split (44/42/42 head dims for t/h/w, interleaved pairs,
+    theta = 1e4) before the attention;
   * joint text-video attention (appendix Table 4, HunyuanVideo-1.5's joint
     attention over video and padded text, masked through segment ids; the
     ~45k-token CogVideoX1.5 joint sequence of Table 3): each sample is
@@ -61,6 +65,7 @@ class Workload:
     kv_len_range: tuple | None = None   # inclusive (lo, hi) per-sample text lengths
     oracle_rows: int | None = None      # per (b, h) query rows the parity check compares
     joint_text: tuple | None = None     # (text_slots, lo, hi): joint text-video segments
+    rope: tuple | None = None           # ((F, Hp, Wp), s0, (d_t, d_h, d_w), theta, interleaved) on Q and K
     description: str = field(default="", compare=False)
 
     @property
@@ -108,6 +113,12 @@ WORKLOADS = {
         "large720", B=1, H=40, D=128, Sq=75600, Skv=75600, seed=1005, latent=(21, 45, 80),
         oracle_rows=4096,
         description="large-DiT 720p self-attention, latent 21x45x80 -> 75600 tokens"),
+    "rope480": Workload(
+        "rope480", B=1, H=12, D=128, Sq=32760, Skv=32760, seed=1002, latent=(21, 30, 52),
+        logit_gain=math.sqrt(3.0), oracle_rows=4096,
+        rope=((21, 30, 52), 0, (44, 42, 42), 10000.0, True),
+        description="small480 with a 3D rotary embedding of Q and K (Wan-style: 44/42/42 dims of t/h/w, "
+                    "interleaved pairs, theta 1e4) before the attention"),
     "joint45k": Workload(
         "joint45k", B=2, H=48, D=64, Sq=45106, Skv=45106, seed=1006, latent=(11, 48, 85),
         joint_text=(226, 16, 226), oracle_rows=4096,

@@ -26,15 +26,29 @@ def _built():
     binding.load()
 
 
-@pytest.mark.parametrize("name", ["tiny", "small480", "cross", "large480", "large720", "joint45k"])
+@pytest.mark.parametrize("name", ["tiny", "small480", "cross", "large480", "large720", "joint45k", "rope480"])
 def test_workload(name):
-    from paper_2609_18077_gb300 import workloads
+    from paper_2609_18077_gb300 import binding, workloads
+    import oracle
     w = workloads.generate(name)
     rows = w["rows"]
     if rows is not None:
         rows = np.ascontiguousarray(rows[:, :ROWS])
-    out, lse = run_gpu(w["q"], w["k"], w["v"], w["scale"], w["kv_lens"], q_seg=w["q_seg"], kv_seg=w["kv_seg"])
-    o_ref, lse_ref = run_oracle(w["q"], w["k"], w["v"], w["scale"], w["kv_lens"], rows, q_seg=w["q_seg"],
+    q, k = w["q"], w["k"]
+    q_ref, k_ref = q, k
+    wl = w["workload"]
+    if wl.rope is not None:
+        # GPU: rotate on the device, then attend; oracle: rotate in fp64, round to
+        # bf16 (nearest even) as the model's tensors are, then attend in fp64
+        grid, s0, dims, theta, inter = wl.rope
+        q = binding.rope3d(q.cuda(), grid, s0, dims, theta, inter)
+        k = binding.rope3d(k.cuda(), grid, s0, dims, theta, inter)
+        q_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(w["q"]), grid, s0, dims, theta, inter)).to(
+            torch.bfloat16)
+        k_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(w["k"]), grid, s0, dims, theta, inter)).to(
+            torch.bfloat16)
+    out, lse = run_gpu(q, k, w["v"], w["scale"], w["kv_lens"], q_seg=w["q_seg"], kv_seg=w["kv_seg"])
+    o_ref, lse_ref = run_oracle(q_ref, k_ref, w["v"], w["scale"], w["kv_lens"], rows, q_seg=w["q_seg"],
                                 kv_seg=w["kv_seg"])
     stats = compare(out, lse, o_ref, lse_ref, rows)
     print(f"{name}: O max {stats[0]:.3e} mean {stats[1]:.3e} LSE rel {stats[2]:.3e}")

@@ -83,6 +83,21 @@ def test_segments_require_ids(lib):
                                      6 * A, 7 * A, 0.1, None) == 0
 
 
+@pytest.mark.parametrize("kw,status", [
+    (dict(x=None), 1), (dict(y=None), 1), (dict(D=7), 1), (dict(D=0), 1), (dict(D=514), 1),
+    (dict(d_t=3), 1), (dict(d_h=-2), 1), (dict(d_t=64, d_h=64, d_w=2), 1), (dict(theta=0.0), 1),
+    (dict(theta=float("nan")), 1), (dict(B=-1), 1), (dict(F=-1), 1), (dict(s0=-1), 1),
+    (dict(x=A + 2), 3), (dict(y=2 * A + 2), 3), (dict(y=A + 64), 1),   # overlapping, not equal
+    (dict(B=0), 0), (dict(S=0), 0),
+])
+def test_rope_validation(lib, kw, status):
+    a = dict(x=A, y=2 * A, B=1, H=1, S=8, D=128, F=2, Hp=2, Wp=2, s0=0, d_t=44, d_h=42, d_w=42, theta=1e4,
+             interleaved=1)
+    a.update(kw)
+    assert lib.vdx_rope3d(a["x"], a["y"], a["B"], a["H"], a["S"], a["D"], a["F"], a["Hp"], a["Wp"], a["s0"],
+                          a["d_t"], a["d_h"], a["d_w"], a["theta"], a["interleaved"], None) == status
+
+
 def test_selftest_limit_validation(lib):
     assert lib.vdx_selftest_wait_timeout(0, None) == 1
     assert lib.vdx_selftest_wait_timeout(10000001, None) == 1
