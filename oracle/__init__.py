@@ -56,6 +56,12 @@ class Oracle:
             ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
             ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int,
             ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
+        lib.oracle_attn_fwd_win3d.restype = ctypes.c_int
+        lib.oracle_attn_fwd_win3d.argtypes = [
+            ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p,
+            ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_double,
+            ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            ctypes.c_void_p, ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p]
         lib.oracle_rope3d.restype = ctypes.c_int
         lib.oracle_rope3d.argtypes = [
             ctypes.c_void_p, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
@@ -124,6 +130,35 @@ class Oracle:
         return (o, lse, pr) if probs else (o, lse)
 
 
+    def attn_fwd_win3d(self, q, k, v, scale, grid, window, neighbourhood=True, rows=None, probs=False):
+        """Windowed 3D attention in fp64 (see oracle.c).
+
+        q, k, v: uint16 [B,H,S,D] with S = F*Hp*Wp tokens of the grid (F, Hp, Wp)
+        in raster order; window = (kt, kh, kw), odd sizes.
+        Returns (o, lse[, probs]) like attn_fwd.
+        """
+        q, k, v = _bits(q), _bits(k), _bits(v)
+        B, H, S, D = q.shape
+        F, Hp, Wp = (int(x) for x in grid)
+        if S != F * Hp * Wp or k.shape != q.shape or v.shape != q.shape:
+            raise ValueError("q, k, v must be [B,H,F*Hp*Wp,D] alike")
+        if rows is None:
+            n, rows_arr = S, None
+        else:
+            rows_arr = np.ascontiguousarray(np.asarray(rows, dtype=np.int32))
+            if rows_arr.ndim != 2 or rows_arr.shape[0] != B * H:
+                raise ValueError("rows must have shape [B*H, n]")
+            n = rows_arr.shape[1]
+        o = np.empty((B, H, n, D), dtype=np.float64)
+        lse = np.empty((B, H, n), dtype=np.float64)
+        pr = np.empty((B, H, n, S), dtype=np.float64) if probs else None
+        rc = self._lib.oracle_attn_fwd_win3d(_ptr(q), _ptr(k), _ptr(v), B, H, F, Hp, Wp, D, float(scale),
+                                             int(window[0]), int(window[1]), int(window[2]), int(bool(neighbourhood)),
+                                             _ptr(rows_arr), n, _ptr(o), _ptr(lse), _ptr(pr))
+        if rc != 0:
+            raise RuntimeError("oracle_attn_fwd_win3d rejected its arguments")
+        return (o, lse, pr) if probs else (o, lse)
+
     def rope3d(self, x, grid, s0, dims, theta, interleaved=True):
         """3D rotary embedding in fp64 (see oracle.c).
 
@@ -164,6 +199,11 @@ def default() -> Oracle:
             build()
         _default = Oracle(LIBRARY)
     return _default
+
+
+def attn_fwd_win3d(q, k, v, scale, grid, window, neighbourhood=True, rows=None, probs=False):
+    """Module-level shortcut for ``default().attn_fwd_win3d``."""
+    return default().attn_fwd_win3d(q, k, v, scale, grid, window, neighbourhood, rows, probs)
 
 
 def rope3d(x, grid, s0, dims, theta, interleaved=True):

@@ -33,6 +33,17 @@
  * the definition above runs over that key set in ascending key order.  A query
  * whose segment owns no key gets o = 0 and lse = -inf.
  *
+ * Windowed 3D attention (oracle_attn_fwd_win3d): appendix Table 4 names the
+ * LTX-2.5 VAE decoder's 3D neighbourhood attention with an 11 x 11 x 11
+ * window.  The S = F*Hp*Wp tokens are a (t, h, w) grid in raster order and a
+ * query attends exactly the keys inside its window: along each axis of
+ * length L with odd window size k, the window of the query at p is
+ *     neighbourhood: [lo, lo + k) with lo = clamp(p - k/2, 0, max(L - k, 0)),
+ *                    cut to [0, L) (shifted inward at the border, so it
+ *                    always spans min(k, L) positions);
+ *     truncated:     [max(p - k/2, 0), min(p + k/2, L - 1)].
+ * The definition above then runs over that key set in ascending key order.
+ *
  * 3D rotary position embedding (oracle_rope3d).  Sec. 2 of the paper
  * ("3D RoPE, 3D VAEs, and flash attention") keeps each model family's own
  * 3D RoPE convention over time, height and width without stating one.  The
@@ -248,6 +259,101 @@ int oracle_attn_fwd_seg(const uint16_t *q, const uint16_t *k, const uint16_t *v,
             if (probs) {
                 double *pr = probs + (size_t)t * Skv;
                 for (int j = 0; j < Skv; ++j)
+                    pr[j] = 0.0;
+                for (int e = 0; e < n; ++e)
+                    pr[idx[e]] = ps[e];
+            }
+        }
+        free(s);
+        free(ps);
+        free(idx);
+    }
+    return failed ? -1 : 0;
+}
+
+/* Window [lo, hi] of position p on an axis of length L, window size k (odd). */
+static void axis_window(int p, int L, int k, int neighbourhood, int *lo, int *hi)
+{
+    if (neighbourhood) {
+        int start = p - k / 2;
+        const int last_start = L - k > 0 ? L - k : 0;
+        if (start < 0)
+            start = 0;
+        if (start > last_start)
+            start = last_start;
+        *lo = start;
+        *hi = start + k - 1 < L - 1 ? start + k - 1 : L - 1;
+    } else {
+        *lo = p - k / 2 > 0 ? p - k / 2 : 0;
+        *hi = p + k / 2 < L - 1 ? p + k / 2 : L - 1;
+    }
+}
+
+/*
+ * Windowed 3D attention over the grid F x Hp x Wp (S = F*Hp*Wp tokens per
+ * sequence, raster order t, h, w), window kt x kh x kw (odd sizes); see the
+ * header.  rows, o, lse, probs as for oracle_attn_fwd.
+ * Returns 0, or -1 on a bad argument or a failed allocation.
+ */
+int oracle_attn_fwd_win3d(const uint16_t *q, const uint16_t *k, const uint16_t *v,
+                          int B, int H, int F, int Hp, int Wp, int D, double scale,
+                          int kt, int kh, int kw, int neighbourhood,
+                          const int32_t *rows, int nrows, double *o, double *lse, double *probs)
+{
+    if (!q || !k || !v || !o || !lse || B < 0 || H < 0 || F < 0 || Hp < 0 || Wp < 0 || D <= 0 ||
+        kt < 1 || kh < 1 || kw < 1 || !(kt & kh & kw & 1))
+        return -1;
+    const long S_l = (long)F * Hp * Wp;
+    if (S_l > 0x7fffffffL)
+        return -1;
+    const int S = (int)S_l;
+    const int nr = rows ? nrows : S;
+    if (nr < 0)
+        return -1;
+    const long total = (long)B * H * nr;
+    const size_t cap = (size_t)(S > 0 ? S : 1);
+    int failed = 0;
+
+#pragma omp parallel
+    {
+        double *s = (double *)malloc(sizeof(double) * cap);
+        double *ps = (double *)malloc(sizeof(double) * cap);
+        int *idx = (int *)malloc(sizeof(int) * cap);
+        if (!s || !ps || !idx) {
+#pragma omp atomic write
+            failed = 1;
+        }
+#pragma omp for schedule(dynamic, 4)
+        for (long t = 0; t < total; ++t) {
+            if (!s || !ps || !idx)
+                continue;
+            const long bh = t / nr;
+            const int r = (int)(t % nr);
+            const int i = rows ? rows[bh * nrows + r] : r;
+            if (i < 0 || i >= S) {
+#pragma omp atomic write
+                failed = 1;
+                continue;
+            }
+            /* the query's grid position and window on each axis */
+            const int pt = i / (Hp * Wp), ph = (i / Wp) % Hp, pw = i % Wp;
+            int tlo, thi, hlo, hhi, wlo, whi;
+            axis_window(pt, F, kt, neighbourhood, &tlo, &thi);
+            axis_window(ph, Hp, kh, neighbourhood, &hlo, &hhi);
+            axis_window(pw, Wp, kw, neighbourhood, &wlo, &whi);
+            /* the keys inside it, in ascending order */
+            int n = 0;
+            for (int tt = tlo; tt <= thi; ++tt)
+                for (int hh = hlo; hh <= hhi; ++hh)
+                    for (int ww = wlo; ww <= whi; ++ww)
+                        idx[n++] = (tt * Hp + hh) * Wp + ww;
+            const uint16_t *qi = q + ((size_t)bh * S + i) * D;
+            const uint16_t *kb = k + (size_t)bh * S * D;
+            const uint16_t *vb = v + (size_t)bh * S * D;
+            attend_row(qi, kb, vb, idx, n, D, scale, s, o + (size_t)t * D, lse + t, probs ? ps : NULL);
+            if (probs) {
+                double *pr = probs + (size_t)t * S;
+                for (int j = 0; j < S; ++j)
                     pr[j] = 0.0;
                 for (int e = 0; e < n; ++e)
                     pr[idx[e]] = ps[e];

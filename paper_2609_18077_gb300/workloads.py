@@ -24,6 +24,11 @@ Recipe (every draw is seeded; no dataset is read):
     [lo, hi]; K/V rows past a sample's length are padding and may be filled
     with NaN to prove they are never read;
   * row subsets for large configs: per (b, h), n distinct query rows;
+  * windowed 3D attention (appendix Table 4: the LTX-2.5 VAE decoder's
+    neighbourhood attention with an 11^3 window): the win3d workload's tokens
+    are a 16x32x48 grid in raster order (t, h, w), each query attending the
+    11x11x11 window around it (shifted inward at the border); the decoder's
+    shapes are not in the paper, so H = 8 and D = 128 are our choice;
   * 3D RoPE (Sec. 2: each family keeps its own convention): the rope480
     workload rotates small480's Q and K over its 21x30x52 grid with Wan's
     published split (44/42/42 head dims for t/h/w, interleaved pairs,
@@ -66,6 +71,7 @@ class Workload:
     oracle_rows: int | None = None      # per (b, h) query rows the parity check compares
     joint_text: tuple | None = None     # (text_slots, lo, hi): joint text-video segments
     rope: tuple | None = None           # ((F, Hp, Wp), s0, (d_t, d_h, d_w), theta, interleaved) on Q and K
+    window: tuple | None = None         # ((kt, kh, kw), neighbourhood): windowed attention over the latent grid
     description: str = field(default="", compare=False)
 
     @property
@@ -88,6 +94,8 @@ class Workload:
         """
         if q_seg is not None:
             return 4.0 * self.H * self.D * float(segment_pairs(q_seg, kv_seg))
+        if self.window is not None:
+            return 4.0 * self.B * self.H * self.D * float(window_pairs(self.latent, *self.window))
         if kv_lens is None:
             return 4.0 * self.B * self.H * self.Sq * self.Skv * self.D
         return 4.0 * self.H * self.Sq * self.D * float(np.sum(np.clip(kv_lens, 0, self.Skv)))
@@ -119,6 +127,11 @@ WORKLOADS = {
         rope=((21, 30, 52), 0, (44, 42, 42), 10000.0, True),
         description="small480 with a 3D rotary embedding of Q and K (Wan-style: 44/42/42 dims of t/h/w, "
                     "interleaved pairs, theta 1e4) before the attention"),
+    "win3d": Workload(
+        "win3d", B=1, H=8, D=128, Sq=24576, Skv=24576, seed=1007, latent=(16, 32, 48),
+        window=((11, 11, 11), True), oracle_rows=4096,
+        description="3D neighbourhood attention with an 11x11x11 window over a 16x32x48 latent grid "
+                    "(the LTX-2.5 VAE decoder's windowed attention; shapes are not in the paper)"),
     "joint45k": Workload(
         "joint45k", B=2, H=48, D=64, Sq=45106, Skv=45106, seed=1006, latent=(11, 48, 85),
         joint_text=(226, 16, 226), oracle_rows=4096,
@@ -190,6 +203,21 @@ def joint_segments(text_lens, text_slots, S) -> np.ndarray:
     for b, L in enumerate(np.asarray(text_lens)):
         seg[b, int(L):text_slots] = 0
     return seg
+
+
+def window_pairs(grid, window, neighbourhood) -> int:
+    """Number of (query, key) pairs inside the windows of one sequence."""
+    total = 1
+    for L, k in zip(grid, window):
+        p = np.arange(L)
+        if neighbourhood:
+            n = min(k, L)
+            total *= n * L
+            continue
+        lo = np.maximum(p - k // 2, 0)
+        hi = np.minimum(p + k // 2, L - 1)
+        total *= int(np.sum(hi - lo + 1))
+    return int(total)
 
 
 def segment_pairs(q_seg, kv_seg) -> int:

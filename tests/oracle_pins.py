@@ -19,6 +19,9 @@ Sources of the facts (none of them is the oracle's own code):
     segment everywhere is dense attention; packed segments are independent
     problems; a prefix segment is the valid-count form; torch's SDPA with the
     boolean mask q_seg[i] == kv_seg[j];
+  * windowed 3D attention: torch SDPA with the window mask (each border rule
+    characterised independently), whole-grid windows as dense attention, a
+    1x1x1 window, window sizes, interior agreement of the two rules;
   * 3D RoPE: the textbook complex form z exp(i phi), norm preservation,
     identity off the grid and at its origin, one axis per coordinate, dot
     products depending on relative position only, and the two pairings
@@ -410,6 +413,84 @@ def pin_rope_pairing_conventions(orc):
     np.testing.assert_allclose(yi, yh[..., perm], rtol=0, atol=1e-13)
 
 
+# ---- windowed 3D attention (appendix Table 4: the LTX-2.5 VAE decoder's 11^3 neighbourhood attention)
+
+def _coords(grid):
+    F, Hp, Wp = grid
+    i = np.arange(F * Hp * Wp)
+    return i // (Hp * Wp), (i // Wp) % Hp, i % Wp
+
+
+def _window_sets(grid, window, neighbourhood):
+    """[S, S] boolean: query i may attend key j.  Independent characterisations:
+    neighbourhood = the in-range run of k positions whose centre is closest to p
+    (brute force over every start); truncated = {j : |j - p| <= k // 2}."""
+    axes = []
+    for p_arr, L, kk in zip(_coords(grid), grid, window):
+        if neighbourhood:
+            n = min(kk, L)
+            starts = np.arange(L - n + 1)
+            best = starts[np.argmin(np.abs(starts[None, :] + (n - 1) / 2.0 - np.arange(L)[:, None]), axis=1)]
+            lo = best[p_arr]
+            ok = (p_arr[None, :] >= lo[:, None]) & (p_arr[None, :] < lo[:, None] + n)
+        else:
+            ok = np.abs(p_arr[None, :] - p_arr[:, None]) <= kk // 2
+        axes.append(ok)
+    return axes[0] & axes[1] & axes[2]
+
+
+def pin_win3d_torch_masked_sdpa(orc):
+    """Both border rules against torch SDPA with the window mask, fp64 (a library)."""
+    grid = (3, 4, 5)
+    S = 60
+    q, k, v = random_qkv(2, 2, S, S, 16, seed=41, logit_gain=1.5)
+    for window, nb in (((3, 3, 3), True), ((3, 3, 3), False), ((1, 3, 5), True), ((3, 1, 3), False)):
+        o, lse = orc.attn_fwd_win3d(bf16_bits(q), bf16_bits(k), bf16_bits(v), 0.3, grid, window, nb)
+        mask = torch.from_numpy(_window_sets(grid, window, nb))
+        qd, kd, vd = q.double(), k.double(), v.double()
+        want = torch.nn.functional.scaled_dot_product_attention(qd, kd, vd, attn_mask=mask, scale=0.3)
+        logits = (0.3 * (qd @ kd.transpose(-1, -2))).masked_fill(~mask, -math.inf)
+        np.testing.assert_allclose(o, want.numpy(), rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse, torch.logsumexp(logits, -1).numpy(), rtol=1e-13, atol=1e-12)
+
+
+def pin_win3d_whole_grid_is_dense(orc):
+    """A window as large as the grid (neighbourhood) or twice as large (truncated) is dense attention."""
+    grid = (2, 3, 4)
+    q, k, v = _inputs(1, 2, 24, 24, 8, seed=42, gain=1.4)
+    o, lse = orc.attn_fwd(q, k, v, 0.5)
+    for window, nb in (((3, 3, 5), True), ((3, 5, 7), False)):
+        ow, lw = orc.attn_fwd_win3d(q, k, v, 0.5, grid, window, nb)
+        np.testing.assert_array_equal(ow, o)
+        np.testing.assert_array_equal(lw, lse)
+
+
+def pin_win3d_single_cell(orc):
+    """A 1 x 1 x 1 window: each query sees only its own key: O = its V, LSE = scale q.k."""
+    grid = (2, 2, 3)
+    q, k, v = _inputs(1, 1, 12, 12, 8, seed=43)
+    o, lse = orc.attn_fwd_win3d(q, k, v, 0.7, grid, (1, 1, 1), True)
+    np.testing.assert_array_equal(o, _dec(v))
+    np.testing.assert_allclose(lse, 0.7 * np.einsum("bhid,bhid->bhi", _dec(q), _dec(k)), rtol=1e-15, atol=1e-14)
+
+
+def pin_win3d_counts_and_interior(orc):
+    """Neighbourhood windows always hold prod(min(k, L)) keys; away from the
+    border both rules give the same window, hence the same result."""
+    grid, window = (5, 6, 7), (3, 3, 5)
+    S = 210
+    q, k, v = _inputs(1, 1, S, S, 8, seed=44, gain=1.2)
+    on, ln, pn = orc.attn_fwd_win3d(q, k, v, 0.4, grid, window, True, probs=True)
+    ot, lt = orc.attn_fwd_win3d(q, k, v, 0.4, grid, window, False)
+    assert np.all(np.count_nonzero(pn[0, 0], axis=1) == 3 * 3 * 5)
+    t, h, w = _coords(grid)
+    inner = (t >= 1) & (t <= 3) & (h >= 1) & (h <= 4) & (w >= 2) & (w <= 4)
+    assert inner.any() and (~inner).any()
+    np.testing.assert_array_equal(on[0, 0, inner], ot[0, 0, inner])
+    np.testing.assert_array_equal(ln[0, 0, inner], lt[0, 0, inner])
+    assert np.any(on[0, 0, ~inner] != ot[0, 0, ~inner])
+
+
 ALL_PINS = [pin_single_key, pin_two_keys, pin_weights_sum_to_one, pin_constant_values,
             pin_zero_logits, pin_query_permutation, pin_key_value_permutation,
             pin_value_translation, pin_varlen_is_truncation, pin_varlen_empty_and_clamped,
@@ -417,4 +498,6 @@ ALL_PINS = [pin_single_key, pin_two_keys, pin_weights_sum_to_one, pin_constant_v
             pin_segments_one_segment_is_dense, pin_segments_packed_are_independent,
             pin_segments_prefix_is_valid_count, pin_segments_torch_masked_sdpa,
             pin_rope_complex_rotation, pin_rope_norm_and_identity, pin_rope_one_axis_each,
-            pin_rope_relative_position, pin_rope_pairing_conventions]
+            pin_rope_relative_position, pin_rope_pairing_conventions,
+            pin_win3d_torch_masked_sdpa, pin_win3d_whole_grid_is_dense, pin_win3d_single_cell,
+            pin_win3d_counts_and_interior]

@@ -53,6 +53,12 @@ MUTANTS = {
                            ("(interleaved ? 2 * i + 1 : i + da / 2)", "(interleaved ? i + da / 2 : 2 * i + 1)")],
     "rope_base_fixed": [("            base += da;\n        }\n    }\n    return 0;", "        }\n    }\n    return 0;")],
     "rope_offset_ignored": [("const long g = s - s0;", "const long g = s;")],
+    "win_h_from_raw_index": [("ph = (i / Wp) % Hp", "ph = i % Hp")],
+    "win_t_from_rows": [("const int pt = i / (Hp * Wp)", "const int pt = i / Wp")],
+    "win_no_inward_shift": [("        if (start > last_start)\n            start = last_start;\n", "")],
+    "win_truncated_radius": [("*hi = p + k / 2 < L - 1 ? p + k / 2 : L - 1;", "*hi = p + k / 2 - 1 < L - 1 ? p + k / 2 - 1 : L - 1;")],
+    "win_key_index_axes": [("idx[n++] = (tt * Hp + hh) * Wp + ww;", "idx[n++] = (tt * Wp + hh) * Hp + ww;")],
+    "win_w_axis_uses_h_size": [("axis_window(pw, Wp, kw,", "axis_window(pw, Wp, kh,")],
 }
 
 CHILD = r"""
