@@ -3,11 +3,13 @@
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
 
 One step = one attention forward (one vdx_attn_fwd / vdx_attn_fwd_varlen /
-vdx_attn_fwd_segments call) over the whole workload, inputs resident in
-HBM.  The default workload is the small-DiT 480p self-attention (B=1, H=12,
+vdx_attn_fwd_segments / vdx_attn_fwd_win3d call, preceded by two
+vdx_rope3d calls for the rope workload) over the whole workload, inputs
+resident in HBM.  The default workload is the small-DiT 480p self-attention (B=1, H=12,
 D=128, S = 21*30*52 = 32760 tokens, logit std ~3).  FLOPs = 4*B*H*Sq*Skv*D
 (effective key counts for the padded-text workload; the (query, key) pairs
-of equal segment id for the joint text-video workload).
+of equal segment id for the joint text-video workload; the (query, key)
+pairs inside the windows for the windowed workload).
 
 Timing: W untimed warm-up steps, then K steps bracketed by a barrier and a
 device synchronisation, timed with CUDA events on the launching stream; the
@@ -156,6 +158,9 @@ def run_ours(args):
     # kernels of ours per step: the segment path builds its key-tile lists first
     launches_per_step = 3 if segs is not None else 1
     mode = "seg" if segs is not None else ("varlen" if lens is not None else "dense")
+    if wl.window is not None:
+        mode = "win"
+        launches_per_step = 2     # key-tile lists, then the attention
     rope = wl.rope
     if rope is not None:
         # the step rotates Q and K into buffers of their own, then attends
@@ -163,7 +168,9 @@ def run_ours(args):
         launches_per_step = 3
 
     def step():
-        if rope is not None:
+        if wl.window is not None:
+            binding.attn_fwd_win3d(q, k, v, wl.latent, wl.window[0], wl.window[1], scale=wl.scale, out=out, lse=lse)
+        elif rope is not None:
             grid, s0, dims, theta, inter = rope
             binding.rope3d(q, grid, s0, dims, theta, inter, out=q_r)
             binding.rope3d(k, grid, s0, dims, theta, inter, out=k_r)
@@ -354,6 +361,8 @@ class OracleTimer:
         keys = wl.Skv if lens is None else float(np.mean(np.clip(lens, 0, wl.Skv)))
         if w["q_seg"] is not None:   # mean keys per query row
             keys = workloads.segment_pairs(w["q_seg"], w["kv_seg"]) / float(wl.B * wl.Sq)
+        if wl.window is not None:
+            keys = workloads.window_pairs(wl.latent, *wl.window) / float(wl.Sq)
         self.flops_per_row = 4.0 * keys * wl.D
         self.bh = wl.B * wl.H
         self.n = 1
@@ -362,8 +371,12 @@ class OracleTimer:
         rows = np.stack([np.sort(self.rng.choice(self.wl.Sq, size=n, replace=False))
                          for _ in range(self.bh)]).astype(np.int32)
         t0 = time.perf_counter()
-        self.orc.attn_fwd(*self.bits, self.wl.scale, kv_lens=self.w["kv_lens"], rows=rows,
-                          q_seg=self.w["q_seg"], kv_seg=self.w["kv_seg"])
+        if self.wl.window is not None:
+            self.orc.attn_fwd_win3d(*self.bits, self.wl.scale, self.wl.latent, self.wl.window[0],
+                                    self.wl.window[1], rows=rows)
+        else:
+            self.orc.attn_fwd(*self.bits, self.wl.scale, kv_lens=self.w["kv_lens"], rows=rows,
+                              q_seg=self.w["q_seg"], kv_seg=self.w["kv_seg"])
         return time.perf_counter() - t0
 
     def calibrate(self, target_s):

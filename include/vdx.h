@@ -108,6 +108,25 @@ int vdx_attn_fwd_segments(const void *q, const void *k, const void *v, void *out
                           float scale, void *stream);
 
 /*
+ * Windowed 3D attention (appendix Table 4: the LTX-2.5 VAE decoder's 3D
+ * neighbourhood attention, an 11 x 11 x 11 window).  As vdx_attn_fwd with
+ * Sq = Skv = S = F*Hp*Wp, the tokens of each sequence being a (t, h, w) grid
+ * in raster order, except that a query attends only the keys inside its
+ * window.  Along an axis of length L with odd window size k (kt, kh, kw), the
+ * window of position p is
+ *   neighbourhood = 1: [lo, min(lo + k, L) - 1], lo = clamp(p - k/2, 0, max(L - k, 0))
+ *                      (shifted inward at the border: always min(k, L) positions);
+ *   neighbourhood = 0: [max(p - k/2, 0), min(p + k/2, L - 1)] (truncated).
+ * Key tiles (128 keys) outside every window of a query-tile pair are skipped;
+ * the rest compare positions element by element.  A small kernel builds the
+ * key-tile lists first, on the same stream, in the library's per-stream
+ * workspace (ceil(S/256) x ceil(S/128) x 4 bytes).
+ */
+int vdx_attn_fwd_win3d(const void *q, const void *k, const void *v, void *out, float *lse,
+                       int B, int H, int F, int Hp, int Wp, int D, int kt, int kh, int kw,
+                       int neighbourhood, float scale, void *stream);
+
+/*
  * 3D rotary position embedding of queries or keys (Sec. 2: each model family
  * keeps its own 3D RoPE convention over time, height and width; this call
  * takes the conventions as parameters).  The standard rotary embedding over a

@@ -33,6 +33,7 @@ SIGNATURES = {
     "vdx_attn_fwd_varlen": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, ctypes.c_float, _P]),
     "vdx_attn_fwd_segments": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, ctypes.c_float, _P]),
     "vdx_attn_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, ctypes.c_float, _P]),
+    "vdx_attn_fwd_win3d": (_I, [_P, _P, _P, _P, _P] + [_I] * 10 + [ctypes.c_float, _P]),
     "vdx_rope3d": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _I, _I, _I, ctypes.c_float, _I, _P]),
     "vdx_status_string": (ctypes.c_char_p, [_I]),
     "vdx_check_device_error": (_I, [_P]),
@@ -208,3 +209,26 @@ def rope3d(x, grid, s0, dims, theta, interleaved=True, out=None):
     if st != VDX_OK:
         raise VdxError(st, "vdx_rope3d")
     return out
+
+
+def attn_fwd_win3d(q, k, v, grid, window, neighbourhood=True, scale=None, out=None, lse=None, return_lse=True):
+    """Windowed 3D attention through ``vdx_attn_fwd_win3d``.
+
+    q, k, v: bf16 [B,H,S,D] with S = F*Hp*Wp tokens of grid = (F, Hp, Wp) in
+    raster order; window = (kt, kh, kw), odd sizes.
+    """
+    _check_qkv(q, k, v)
+    B, H, S, D = q.shape
+    F, Hp, Wp = (int(x) for x in grid)
+    if S != F * Hp * Wp or k.shape[2] != S:
+        raise ValueError(f"q, k, v must hold the F*Hp*Wp = {F * Hp * Wp} grid tokens")
+    scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
+    out, lse = _outputs(q, out, lse, return_lse)
+    with torch.cuda.device(q.device):
+        st = load().vdx_attn_fwd_win3d(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                                       lse.data_ptr() if lse is not None else None, B, H, F, Hp, Wp, D,
+                                       int(window[0]), int(window[1]), int(window[2]), int(bool(neighbourhood)),
+                                       scale, _stream_handle(q.device))
+    if st != VDX_OK:
+        raise VdxError(st, "vdx_attn_fwd_win3d")
+    return out, lse

@@ -60,6 +60,7 @@
 
 #include "segment_tiles.cuh"
 #include "sm103_ptx.cuh"
+#include "window_tiles.cuh"
 
 namespace vdx {
 
@@ -67,6 +68,9 @@ namespace vdx {
 constexpr int MODE_DENSE = 0;    // all Skv keys
 constexpr int MODE_VARLEN = 1;   // the first kv_lens[b] keys of sample b
 constexpr int MODE_SEG = 2;      // the keys whose segment id equals the query's
+constexpr int MODE_WIN = 3;      // the keys inside the query's 3D window (S = F*Hp*Wp grid tokens)
+// Modes that visit key tiles from a list and may mask a row's every key so far.
+__host__ __device__ constexpr bool listed(int mode) { return mode == MODE_SEG || mode == MODE_WIN; }
 
 // Device error word: bit 0 = a bounded wait expired.  Read and cleared by
 // vdx_check_device_error.
@@ -114,6 +118,7 @@ struct SegParams {
     const uint32_t *tlist;
     const int *tcount;
     int n_kt;             // key tiles of the whole sequence, ceil(Skv / BN)
+    WinGrid win;          // MODE_WIN: grid and window; lists per query-tile pair, shared by (b, h)
 };
 
 // Shared-memory plan.  QBUF Q-tile pairs (2 = the next item's Q tiles load
@@ -405,8 +410,8 @@ __device__ __forceinline__ Item unit_item(const AttnParams &p, const SegParams &
         w.kv_valid = len < 0 ? 0 : (len > p.Skv ? p.Skv : len);
     }
     w.n_kv = (w.kv_valid + BN - 1) / BN;
-    if (MODE == MODE_SEG) {
-        const int pair = (w.bh / p.H) * p.q_pairs + w.qp;
+    if (listed(MODE)) {
+        const int pair = MODE == MODE_WIN ? w.qp : (w.bh / p.H) * p.q_pairs + w.qp;
         w.n_kv = __ldg(sp.tcount + pair);
         w.list_off = pair * sp.n_kt;
     }
@@ -451,7 +456,7 @@ __device__ __forceinline__ Item item_at(const AttnParams &p, const SegParams &sp
 template <int MODE>
 __device__ __forceinline__ uint32_t tile_entry(const SegParams &sp, const Item &w, int r)
 {
-    if (MODE == MODE_SEG)
+    if (listed(MODE))
         return __ldg(sp.tlist + w.list_off + r);
     return static_cast<uint32_t>(r);
 }
@@ -569,7 +574,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             if (lane == 0) {
                 const uint32_t bytes = ((has_v && !fix) + has_k) * L::TILE_BYTES;
-                if (MODE == MODE_SEG && has_v)
+                if (listed(MODE) && has_v)
                     reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF)[st] = ventry;
                 if (bytes) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_FULL + st), bytes);
@@ -768,20 +773,37 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     break;
                 ptx::tc_fence_after_sync();
                 const int gj = g + (j - w.j0);
+                // MODE_WIN: the list entry comes with the stage's full barrier, so
+                // that wait comes first here; the row's 128-key window mask is
+                // then built while the logits are not yet in registers.
+                uint32_t wmask[4] = {0u, 0u, 0u, 0u};
+                bool win_mask = false;
+                int kt_win = j;
+                if (MODE == MODE_WIN) {
+                    if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + gj % L::NSTAGE),
+                                                                    (gj / L::NSTAGE) & 1, abort_flag, limit))))
+                        break;
+                    const uint32_t entry = reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF)[gj % L::NSTAGE];
+                    kt_win = static_cast<int>(entry & SEG_TILE_BITS);
+                    win_mask = (entry >> (SEG_MASK_SHIFT + t)) & 1u;
+                    if (win_mask)
+                        window_mask(sp.win, p.Sq, store ? q_row : 0, kt_win, wmask);
+                }
                 uint32_t s[4][32];
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
                     ptx::tmem_ld32(s_addr + 32 * c, s[c]);
                 // The stage (V_j, next K) must have landed before P_t(j) is
                 // published; checked here, under the TMEM load latency.
-                if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + gj % L::NSTAGE),
+                if (MODE != MODE_WIN &&
+                    !(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + gj % L::NSTAGE),
                                                                 (gj / L::NSTAGE) & 1, abort_flag, limit)))) {
                     ptx::tmem_wait_ld();
                     break;
                 }
                 ptx::tmem_wait_ld();
 
-                int kt = j;   // key tile
+                int kt = MODE == MODE_WIN ? kt_win : j;   // key tile
                 bool seg_mask = false;
                 if (MODE == MODE_SEG) {
                     // the stage's list entry, published with its full barrier
@@ -821,6 +843,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         s[c >> 5][c & 31] = kid == my_seg ? s[c >> 5][c & 31] : pad;
                     }
                 }
+                if (MODE == MODE_WIN && win_mask) {
+                    // keys outside this row's window get the masked logit
+                    const uint32_t pad = neg_scale ? 0x7F800000u : 0xFF800000u;
+#pragma unroll
+                    for (int c = 0; c < BN; ++c)
+                        s[c >> 5][c & 31] = (wmask[c >> 5] >> (c & 31)) & 1u ? s[c >> 5][c & 31] : pad;
+                }
                 const float ext = row_extreme(s, neg_scale);
                 const float m_tile = ext * sl2;
                 const float m_new = fmaxf(m_used, m_tile);
@@ -832,7 +861,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 // MODE_SEG: a row whose keys so far were all masked keeps
                 // m_used = -inf; its weights are 2^-inf = 0, not 2^(-inf + inf).
-                const float neg_m = (MODE == MODE_SEG && m_used == -INFINITY) ? 0.f : -m_used;
+                const float neg_m = (listed(MODE) && m_used == -INFINITY) ? 0.f : -m_used;
                 // the tile's largest weight, computed exactly as in row_probs
                 const float p_top = ex2(fmaf(ext, sl2, neg_m));
                 l_exact *= factor;
@@ -894,7 +923,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                     bar(L::B_MERGE + 1), abort_flag);
             } else {
                 // MODE_SEG: a row with no key of its segment has l = 0 and O = 0.
-                const float inv_l = (MODE == MODE_SEG && !(l_exact > 0.f)) ? 0.f : 1.f / (l_exact + l_resid);
+                const float inv_l = (listed(MODE) && !(l_exact > 0.f)) ? 0.f : 1.f / (l_exact + l_resid);
                 uint32_t w16[D / 32][16];
 #pragma unroll
                 for (int c = 0; c < D / 32; ++c) {

@@ -72,8 +72,9 @@ cudaError_t raise_all_smem_limits()
     cudaError_t e = cudaSuccess;
     using namespace vdx;
     for (cudaError_t r : {raise_smem_limit<128, MODE_DENSE, 1, 2>(), raise_smem_limit<128, MODE_VARLEN, 1, 2>(),
-                          raise_smem_limit<128, MODE_SEG, 1, 2>(), raise_smem_limit<64, MODE_DENSE, 2, 4>(),
-                          raise_smem_limit<64, MODE_VARLEN, 2, 4>(), raise_smem_limit<64, MODE_SEG, 2, 4>()})
+                          raise_smem_limit<128, MODE_SEG, 1, 2>(), raise_smem_limit<128, MODE_WIN, 1, 2>(),
+                          raise_smem_limit<64, MODE_DENSE, 2, 4>(), raise_smem_limit<64, MODE_VARLEN, 2, 4>(),
+                          raise_smem_limit<64, MODE_SEG, 2, 4>(), raise_smem_limit<64, MODE_WIN, 2, 4>()})
         if (r != cudaSuccess)
             e = r;
     return e;
@@ -184,6 +185,7 @@ struct KeyRule {
     const int *kv_lens = nullptr;
     const int *q_seg = nullptr;
     const int *kv_seg = nullptr;
+    vdx::WinGrid win{};   // MODE_WIN
 };
 
 // fixed_scratch / fixed_bytes: when set, the split-tail workspace is taken
@@ -194,6 +196,7 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
 {
     const bool varlen = rule.mode == vdx::MODE_VARLEN;
     const bool seg = rule.mode == vdx::MODE_SEG;
+    const bool win = rule.mode == vdx::MODE_WIN;
     const int *kv_lens = rule.kv_lens;
     // ---- validation (no CUDA calls)
     if (!q || !k || !v || !out || (varlen && !kv_lens) || (seg && (!rule.q_seg || !rule.kv_seg)))
@@ -328,18 +331,42 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         sp.tcount = tcount;
         sp.n_kt = n_kv;
     }
+    if (win) {
+        // Key-tile lists per query-tile pair, shared by every (b, h).
+        const size_t list_bytes = round_up(static_cast<size_t>(q_pairs) * n_kv * 4, 256);
+        const size_t cnt_bytes = round_up(static_cast<size_t>(q_pairs) * 4, 256);
+        int dev = 0;
+        void *ws = nullptr;
+        if (cudaGetDevice(&dev) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        if ((st = workspace(dev, s, list_bytes + cnt_bytes, &ws)) != VDX_OK)
+            return st;
+        uint32_t *tlist = static_cast<uint32_t *>(ws);
+        int *tcount = reinterpret_cast<int *>(static_cast<char *>(ws) + list_bytes);
+        vdx::win_tile_lists_kernel<<<static_cast<unsigned>((q_pairs + 7) / 8), 256, 0, s>>>(
+            rule.win, Sq, static_cast<int>(q_pairs), n_kv, tlist, tcount);
+        if (cudaGetLastError() != cudaSuccess)
+            return VDX_ERR_CUDA;
+        sp.tlist = tlist;
+        sp.tcount = tcount;
+        sp.n_kt = n_kv;
+        sp.win = rule.win;
+    }
     using vdx::MODE_DENSE;
     using vdx::MODE_SEG;
     using vdx::MODE_VARLEN;
+    using vdx::MODE_WIN;
     cudaError_t e;
     if (D == 128) {
         e = varlen ? launch<128, MODE_VARLEN, 1, 2>(grid, mq, mk, mv, p, sp, s)
                    : seg ? launch<128, MODE_SEG, 1, 2>(grid, mq, mk, mv, p, sp, s)
-                         : launch<128, MODE_DENSE, 1, 2>(grid, mq, mk, mv, p, sp, s);
+                         : win ? launch<128, MODE_WIN, 1, 2>(grid, mq, mk, mv, p, sp, s)
+                               : launch<128, MODE_DENSE, 1, 2>(grid, mq, mk, mv, p, sp, s);
     } else {
         e = varlen ? launch<64, MODE_VARLEN, 2, 4>(grid, mq, mk, mv, p, sp, s)
                    : seg ? launch<64, MODE_SEG, 2, 4>(grid, mq, mk, mv, p, sp, s)
-                         : launch<64, MODE_DENSE, 2, 4>(grid, mq, mk, mv, p, sp, s);
+                         : win ? launch<64, MODE_WIN, 2, 4>(grid, mq, mk, mv, p, sp, s)
+                               : launch<64, MODE_DENSE, 2, 4>(grid, mq, mk, mv, p, sp, s);
     }
     if (e == cudaErrorNoKernelImageForDevice)
         return VDX_ERR_DEVICE;
@@ -421,6 +448,26 @@ int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, 
     rule.mode = vdx::MODE_VARLEN;
     rule.kv_lens = kv_lens;
     return attn_launch(q, k, v, out, lse, B, H, Sq, Skv_max, D, rule, scale, stream);
+}
+
+int vdx_attn_fwd_win3d(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int F,
+                       int Hp, int Wp, int D, int kt, int kh, int kw, int neighbourhood, float scale, void *stream)
+{
+    if (F < 0 || Hp < 0 || Wp < 0 || kt < 1 || kh < 1 || kw < 1 || !(kt & kh & kw & 1))
+        return VDX_ERR_INVALID_ARG;
+    const long long S = static_cast<long long>(F) * Hp * Wp;
+    if (S > INT_MAX)
+        return VDX_ERR_UNSUPPORTED;
+    KeyRule rule;
+    rule.mode = vdx::MODE_WIN;
+    rule.win.F = F;
+    rule.win.Hp = Hp;
+    rule.win.Wp = Wp;
+    rule.win.kt = kt;
+    rule.win.kh = kh;
+    rule.win.kw = kw;
+    rule.win.neighbourhood = neighbourhood ? 1 : 0;
+    return attn_launch(q, k, v, out, lse, B, H, static_cast<int>(S), static_cast<int>(S), D, rule, scale, stream);
 }
 
 int vdx_rope3d(const void *x, void *y, int B, int H, int S, int D, int F, int Hp, int Wp, int s0, int d_t, int d_h,

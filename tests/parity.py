@@ -54,9 +54,13 @@ def compare(o_gpu, lse_gpu, o_ref, lse_ref, rows=None):
     return max_abs, mean_abs, lse_rel
 
 
-def run_gpu(q, k, v, scale, kv_lens=None, device="cuda", with_lse=True, q_seg=None, kv_seg=None):
+def run_gpu(q, k, v, scale, kv_lens=None, device="cuda", with_lse=True, q_seg=None, kv_seg=None, window=None):
+    """window: None or (grid, (kt, kh, kw), neighbourhood) for windowed 3D attention."""
     qd, kd, vd = (t.to(device) for t in (q, k, v))
-    if q_seg is not None:
+    if window is not None:
+        grid, ks, nb = window
+        out, lse = binding.attn_fwd_win3d(qd, kd, vd, grid, ks, nb, scale=scale, return_lse=with_lse)
+    elif q_seg is not None:
         qs = torch.from_numpy(np.ascontiguousarray(q_seg, dtype=np.int32)).to(device)
         ks = torch.from_numpy(np.ascontiguousarray(kv_seg, dtype=np.int32)).to(device)
         out, lse = binding.attn_fwd_segments(qd, kd, vd, qs, ks, scale=scale, return_lse=with_lse)
@@ -70,7 +74,11 @@ def run_gpu(q, k, v, scale, kv_lens=None, device="cuda", with_lse=True, q_seg=No
     return out, lse
 
 
-def run_oracle(q, k, v, scale, kv_lens=None, rows=None, q_seg=None, kv_seg=None):
+def run_oracle(q, k, v, scale, kv_lens=None, rows=None, q_seg=None, kv_seg=None, window=None):
+    if window is not None:
+        grid, ks, nb = window
+        return oracle.attn_fwd_win3d(workloads.bf16_bits(q), workloads.bf16_bits(k), workloads.bf16_bits(v),
+                                     scale, grid, ks, nb, rows=rows)
     return oracle.attn_fwd(workloads.bf16_bits(q), workloads.bf16_bits(k), workloads.bf16_bits(v),
                            scale, kv_lens=kv_lens, rows=rows, q_seg=q_seg, kv_seg=kv_seg)
 

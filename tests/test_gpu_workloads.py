@@ -26,7 +26,8 @@ def _built():
     binding.load()
 
 
-@pytest.mark.parametrize("name", ["tiny", "small480", "cross", "large480", "large720", "joint45k", "rope480"])
+@pytest.mark.parametrize("name", ["tiny", "small480", "cross", "large480", "large720", "joint45k", "rope480",
+                                  "win3d"])
 def test_workload(name):
     from paper_2609_18077_gb300 import binding, workloads
     import oracle
@@ -47,9 +48,11 @@ def test_workload(name):
             torch.bfloat16)
         k_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(w["k"]), grid, s0, dims, theta, inter)).to(
             torch.bfloat16)
-    out, lse = run_gpu(q, k, w["v"], w["scale"], w["kv_lens"], q_seg=w["q_seg"], kv_seg=w["kv_seg"])
+    window = None if wl.window is None else (wl.latent, wl.window[0], wl.window[1])
+    out, lse = run_gpu(q, k, w["v"], w["scale"], w["kv_lens"], q_seg=w["q_seg"], kv_seg=w["kv_seg"],
+                       window=window)
     o_ref, lse_ref = run_oracle(q_ref, k_ref, w["v"], w["scale"], w["kv_lens"], rows, q_seg=w["q_seg"],
-                                kv_seg=w["kv_seg"])
+                                kv_seg=w["kv_seg"], window=window)
     stats = compare(out, lse, o_ref, lse_ref, rows)
     print(f"{name}: O max {stats[0]:.3e} mean {stats[1]:.3e} LSE rel {stats[2]:.3e}")
     del out, lse

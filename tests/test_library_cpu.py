@@ -98,6 +98,17 @@ def test_rope_validation(lib, kw, status):
                           a["d_t"], a["d_h"], a["d_w"], a["theta"], a["interleaved"], None) == status
 
 
+def test_window_validation(lib):
+    g = GOOD
+    args = (g["q"], g["k"], g["v"], g["out"], g["lse"], 1, 1)
+    assert lib.vdx_attn_fwd_win3d(*args, 2, 2, 2, 128, 4, 3, 3, 1, 0.1, None) == 1      # even window
+    assert lib.vdx_attn_fwd_win3d(*args, 2, 2, 2, 128, 3, 0, 3, 1, 0.1, None) == 1      # empty window
+    assert lib.vdx_attn_fwd_win3d(*args, -1, 2, 2, 128, 3, 3, 3, 1, 0.1, None) == 1
+    assert lib.vdx_attn_fwd_win3d(*args, 2, 2, 2, 96, 3, 3, 3, 1, 0.1, None) == 1       # bad D
+    assert lib.vdx_attn_fwd_win3d(*args, 70000, 70000, 2, 128, 3, 3, 3, 1, 0.1, None) == 2
+    assert lib.vdx_attn_fwd_win3d(*args, 0, 2, 2, 128, 3, 3, 3, 1, 0.1, None) == 0       # no tokens
+
+
 def test_selftest_limit_validation(lib):
     assert lib.vdx_selftest_wait_timeout(0, None) == 1
     assert lib.vdx_selftest_wait_timeout(10000001, None) == 1
