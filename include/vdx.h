@@ -120,7 +120,8 @@ int vdx_attn_fwd_segments(const void *q, const void *k, const void *v, void *out
  * Key tiles (128 keys) outside every window of a query-tile pair are skipped;
  * the rest compare positions element by element.  A small kernel builds the
  * key-tile lists first, on the same stream, in the library's per-stream
- * workspace (ceil(S/256) x ceil(S/128) x 4 bytes).
+ * workspace (ceil(S/256) x ceil(S/128) x 4 bytes).  Grid sides up to 65535;
+ * VDX_ERR_UNSUPPORTED beyond.
  */
 int vdx_attn_fwd_win3d(const void *q, const void *k, const void *v, void *out, float *lse,
                        int B, int H, int F, int Hp, int Wp, int D, int kt, int kh, int kw,

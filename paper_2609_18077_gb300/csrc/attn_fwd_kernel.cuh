@@ -148,10 +148,12 @@ struct Layout {
     static constexpr int TMEM_PTR_OFF = BAR_OFF + NBARS * 8;
     static constexpr int ABORT_OFF = TMEM_PTR_OFF + 4;
     static constexpr int MERGE_OFF = ABORT_OFF + 4;          // "this CTA merges" flag
-    static constexpr int ENTRY_OFF = MERGE_OFF + 4;          // [NSTAGE] MODE_SEG: list entry of each stage's V tile
+    // [NSTAGE][4] listed modes: list entry of each stage's V tile; MODE_WIN also
+    // the grid position of its first key (t | h << 16, w)
+    static constexpr int ENTRY_OFF = (MERGE_OFF + 4 + 15) / 16 * 16;
     // 197.8 KB in all configurations: under the 196 KB shared-memory carve-out
     // (199,680 usable bytes), which leaves 60 KB of L1 for the spill slots.
-    static constexpr int BYTES = ENTRY_OFF + 4 * NSTAGE;
+    static constexpr int BYTES = ENTRY_OFF + 16 * NSTAGE;
     static constexpr int ALLOC = BYTES + 1024;               // slack for 1024-B alignment
 };
 
@@ -574,8 +576,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             if (lane == 0) {
                 const uint32_t bytes = ((has_v && !fix) + has_k) * L::TILE_BYTES;
-                if (listed(MODE) && has_v)
-                    reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF)[st] = ventry;
+                if (listed(MODE) && has_v) {
+                    volatile uint32_t *slot = reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF) + 4 * st;
+                    slot[0] = ventry;
+                    if (MODE == MODE_WIN) {
+                        int t0, h0, w0;
+                        grid_pos(sp.win, vj * BN, t0, h0, w0);
+                        slot[1] = static_cast<uint32_t>(t0) | (static_cast<uint32_t>(h0) << 16);
+                        slot[2] = static_cast<uint32_t>(w0);
+                    }
+                }
                 if (bytes) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_FULL + st), bytes);
                     for (int h = 0; h < D / 64; ++h) {
@@ -768,6 +778,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             float m_used = -INFINITY;
             float l_exact = 0.f;   // sum of the fp32 weights: the log-sum-exp
             float l_resid = 0.f;   // sum over tiles of r - p for each tile's largest weight
+            // MODE_WIN: this row's window, one packed axis per word, for the whole unit
+            uint32_t win_t = 0, win_h = 0, win_w = 0;
+            if (MODE == MODE_WIN)
+                packed_window(sp.win, store ? q_row : 0, win_t, win_h, win_w);
             for (int j = w.j0; j < w.j1; ++j, ++sc) {
                 if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_S + t), sc & 1, abort_flag, limit))))
                     break;
@@ -783,11 +797,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + gj % L::NSTAGE),
                                                                     (gj / L::NSTAGE) & 1, abort_flag, limit))))
                         break;
-                    const uint32_t entry = reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF)[gj % L::NSTAGE];
+                    const volatile uint32_t *slot =
+                        reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF) + 4 * (gj % L::NSTAGE);
+                    const uint32_t entry = slot[0];
                     kt_win = static_cast<int>(entry & SEG_TILE_BITS);
                     win_mask = (entry >> (SEG_MASK_SHIFT + t)) & 1u;
-                    if (win_mask)
-                        window_mask(sp.win, p.Sq, store ? q_row : 0, kt_win, wmask);
+                    if (win_mask) {
+                        const uint32_t th = slot[1];
+                        window_mask(sp.win, p.Sq, win_t, win_h, win_w, kt_win, static_cast<int>(th & 0xFFFFu),
+                                    static_cast<int>(th >> 16), static_cast<int>(slot[2]), wmask);
+                    }
                 }
                 uint32_t s[4][32];
 #pragma unroll
@@ -807,7 +826,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 bool seg_mask = false;
                 if (MODE == MODE_SEG) {
                     // the stage's list entry, published with its full barrier
-                    const uint32_t entry = reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF)[gj % L::NSTAGE];
+                    const uint32_t entry = reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF)[4 * (gj % L::NSTAGE)];
                     kt = static_cast<int>(entry & SEG_TILE_BITS);
                     seg_mask = (entry >> (SEG_MASK_SHIFT + t)) & 1u;
                 }

@@ -456,7 +456,7 @@ int vdx_attn_fwd_win3d(const void *q, const void *k, const void *v, void *out, f
     if (F < 0 || Hp < 0 || Wp < 0 || kt < 1 || kh < 1 || kw < 1 || !(kt & kh & kw & 1))
         return VDX_ERR_INVALID_ARG;
     const long long S = static_cast<long long>(F) * Hp * Wp;
-    if (S > INT_MAX)
+    if (S > INT_MAX || F > 65535 || Hp > 65535 || Wp > 65535)   // window bounds are packed in 16 bits
         return VDX_ERR_UNSUPPORTED;
     KeyRule rule;
     rule.mode = vdx::MODE_WIN;

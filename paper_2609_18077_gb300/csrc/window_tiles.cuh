@@ -169,21 +169,32 @@ __device__ __forceinline__ void set_bit_range(uint32_t (&m)[4], int lo, int hi)
     }
 }
 
-// 128-bit mask of the keys of key tile kt inside the window of query token q:
-// the tile's keys run through (t, h) rows of the grid; per row, the keys whose
-// w lies inside the window form one range.
-__device__ __forceinline__ void window_mask(const WinGrid &g, int S, int q, int kt, uint32_t (&m)[4])
+// The window of query token q, one axis per word: lo in the low 16 bits, hi in
+// the high 16 (grid sides below 65536).
+__device__ __forceinline__ void packed_window(const WinGrid &g, int q, uint32_t &tw, uint32_t &hw, uint32_t &ww)
+{
+    int qt, qh, qw, lo, hi;
+    grid_pos(g, q, qt, qh, qw);
+    axis_window(qt, g.F, g.kt, g.neighbourhood, lo, hi);
+    tw = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
+    axis_window(qh, g.Hp, g.kh, g.neighbourhood, lo, hi);
+    hw = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
+    axis_window(qw, g.Wp, g.kw, g.neighbourhood, lo, hi);
+    ww = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
+}
+
+// 128-bit mask of the keys of key tile kt inside a query's window (packed as
+// above), given the grid position (t, h, w) of the tile's first key: the
+// tile's keys run through (t, h) rows of the grid; per row, the keys whose w
+// lies inside the window form one range.
+__device__ __forceinline__ void window_mask(const WinGrid &g, int S, uint32_t tw, uint32_t hw, uint32_t ww, int kt,
+                                            int t, int h, int w, uint32_t (&m)[4])
 {
     m[0] = m[1] = m[2] = m[3] = 0u;
-    int qt, qh, qw, tlo, thi, hlo, hhi, wlo, whi;
-    grid_pos(g, q, qt, qh, qw);
-    axis_window(qt, g.F, g.kt, g.neighbourhood, tlo, thi);
-    axis_window(qh, g.Hp, g.kh, g.neighbourhood, hlo, hhi);
-    axis_window(qw, g.Wp, g.kw, g.neighbourhood, wlo, whi);
-    const int c0 = kt * 128;
-    const int kn = min(128, S - c0);
-    int t, h, w;
-    grid_pos(g, c0, t, h, w);
+    const int tlo = static_cast<int>(tw & 0xFFFFu), thi = static_cast<int>(tw >> 16);
+    const int hlo = static_cast<int>(hw & 0xFFFFu), hhi = static_cast<int>(hw >> 16);
+    const int wlo = static_cast<int>(ww & 0xFFFFu), whi = static_cast<int>(ww >> 16);
+    const int kn = min(128, S - kt * 128);
     for (int c = 0; c < kn;) {
         const int len = min(g.Wp - w, kn - c);
         if (t >= tlo && t <= thi && h >= hlo && h <= hhi) {
