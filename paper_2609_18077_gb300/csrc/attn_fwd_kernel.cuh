@@ -638,6 +638,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             nw.ok = false;
             if (ni >= 0)
                 nw = item_at<MODE>(p, sp, cta, ni);
+            // The next item's Q tiles can load only once this item's last QK^T
+            // ran; start bringing them to L2 now so that load is short (a hint:
+            // nothing waits for it).
+            if (lane == 0 && nw.ok)
+                for (int t = 0; t < 2; ++t)
+                    for (int h = 0; h < D / 64; ++h)
+                        ptx::tma_prefetch_3d(&tmap_q, h * 64, (nw.qp * 2 + t) * BM, nw.bh);
             uint32_t ve = tile_entry<MODE>(sp, w, w.j0);
             for (int j = w.j0; ok && j < w.j1; ++j) {
                 const bool last = j + 1 == w.j1;
