@@ -174,6 +174,38 @@ int vdx_rope3d(const void *x, void *y, int B, int H, int S, int D, int F, int Hp
 int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out, float *lse,
                          int B, int H, int Sq, int Skv, int D, float scale, void *stream);
 
+/*
+ * Attention forward on HOST buffers (a library service around Sec. 2's
+ * attention op; the paper has no counterpart): vdx_attn_fwd, or
+ * vdx_attn_fwd_varlen when kv_lens != NULL, for callers whose tensors live in
+ * host memory.  The library copies the inputs in, runs the kernel and copies
+ * the results out, overlapping the three: the (b, h) rows are cut into
+ * chunks, and chunk i's kernel runs while chunk i+1 is copied in and chunk
+ * i-1 copied out, on two copy streams of the library's own.
+ *   q, k, v, out, lse, kv_lens : HOST pointers, caller-owned, laid out as in
+ *          vdx_attn_fwd(_varlen) (kv_lens: int32 [B], read by the host during
+ *          the call and copied in); lse may be NULL.  No alignment rule.  out
+ *          and lse must not overlap each other or the inputs.
+ *   chunk_rows : (b, h) rows per chunk; 0 lets the library choose from a
+ *          cost model of the copies and the kernel.  With kv_lens, a chunk
+ *          holds heads of one sample or whole samples (rounded down to a
+ *          multiple of H above H).
+ * Ordered after earlier work on `stream`, and `stream` waits for the last
+ * copy out, so out and lse are complete once `stream` is synchronised; the
+ * call itself returns once everything is enqueued.  Copies overlap only when
+ * the host buffers are pinned (page-locked); pageable buffers give the same
+ * results with the copies serialised by the CUDA runtime.  The host buffers
+ * must stay valid until `stream` is synchronised.
+ * Memory: per (device, stream), two device slots of one chunk's q, k, v, out
+ * and lse each (~270 MB for B=1, H=12, S=32760, D=128 at the default
+ * chunking), allocated by the first call, grown by a larger one (which waits
+ * for the device), kept until the process exits; plus vdx_attn_fwd's
+ * workspace.  Errors: as vdx_attn_fwd; chunk_rows < 0 is VDX_ERR_INVALID_ARG.
+ */
+int vdx_attn_fwd_host(const void *q, const void *k, const void *v, void *out, float *lse,
+                      int B, int H, int Sq, int Skv, int D, const int *kv_lens, float scale,
+                      long long chunk_rows, void *stream);
+
 /* Human-readable name of a vdx_status (static storage; never NULL). */
 const char *vdx_status_string(int status);
 

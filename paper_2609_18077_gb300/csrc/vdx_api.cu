@@ -16,6 +16,7 @@
 #include <map>
 #include <mutex>
 #include <utility>
+#include <vector>
 
 #include "attn_fwd_kernel.cuh"
 #include "rope3d.cuh"
@@ -412,6 +413,194 @@ int noalloc_scratch(void **ptr)
     return st.status;
 }
 
+// ---------------------------------------------------------------- host-buffer pipeline
+// vdx_attn_fwd_host cuts the (b, h) rows into chunks.  Chunk i is copied in
+// on one stream, run on one of two compute streams (alternating, so that
+// chunk i+1's CTAs take the multiprocessors that chunk i's last short round
+// leaves idle) and copied out on a third.  kHostSlots device slots (inputs
+// and outputs of one chunk each) rotate over the chunks; events order the
+// reuse of a slot.  One pipeline per (device, caller stream), made by its
+// first call, grown when a call needs larger slots (the old slots are freed,
+// which waits for the device), kept until exit.
+constexpr int kHostSlots = 3;
+
+struct HostPipe {
+    std::mutex mutex;   // one call at a time enqueues on a pipeline
+    bool ready = false;
+    cudaStream_t up = nullptr, down = nullptr, run[2] = {};
+    cudaEvent_t start = nullptr, h2d[kHostSlots] = {}, comp[kHostSlots] = {}, d2h[kHostSlots] = {};
+    void *buf = nullptr;
+    size_t bytes = 0;
+};
+std::mutex g_pipes_mutex;
+std::map<std::pair<int, cudaStream_t>, HostPipe> g_pipes;
+
+HostPipe &host_pipe(int dev, cudaStream_t s)
+{
+    std::lock_guard<std::mutex> lock(g_pipes_mutex);
+    return g_pipes[{dev, s}];   // map nodes never move
+}
+
+int host_pipe_init(HostPipe &pp)
+{
+    if (pp.ready)
+        return VDX_OK;
+    if (cudaStreamCreateWithFlags(&pp.up, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&pp.down, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&pp.run[0], cudaStreamNonBlocking) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&pp.run[1], cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&pp.start, cudaEventDisableTiming) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    for (int i = 0; i < kHostSlots; ++i)
+        if (cudaEventCreateWithFlags(&pp.h2d[i], cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&pp.comp[i], cudaEventDisableTiming) != cudaSuccess ||
+            cudaEventCreateWithFlags(&pp.d2h[i], cudaEventDisableTiming) != cudaSuccess)
+            return VDX_ERR_CUDA;
+    pp.ready = true;
+    return VDX_OK;
+}
+
+// A chunk: rows [row0, row0 + rows) of the flattened (b, h) rows, launched as
+// B x H = nb x nh; its valid key counts start at kv_lens[lens0].
+struct HostChunk {
+    long long row0;
+    int rows, nb, nh;
+    long long lens0;
+};
+
+// Chunks of r rows; varlen chunks hold heads of one sample (r <= H) or whole
+// samples (r a multiple of H), so that one kv_lens offset serves a launch.
+std::vector<HostChunk> make_chunks(long long r, int B, int H, bool varlen)
+{
+    std::vector<HostChunk> chunks;
+    const long long bh = static_cast<long long>(B) * H;
+    if (!varlen) {
+        for (long long r0 = 0; r0 < bh; r0 += r) {
+            const int n = static_cast<int>(bh - r0 < r ? bh - r0 : r);
+            chunks.push_back({r0, n, 1, n, 0});
+        }
+    } else if (r <= H) {
+        for (int b = 0; b < B; ++b)
+            for (int h0 = 0; h0 < H; h0 += static_cast<int>(r)) {
+                const int n = static_cast<int>(H - h0 < r ? H - h0 : r);
+                chunks.push_back({static_cast<long long>(b) * H + h0, n, 1, n, b});
+            }
+    } else {
+        const int per = static_cast<int>(r / H);
+        for (int b0 = 0; b0 < B; b0 += per) {
+            const int nb = B - b0 < per ? B - b0 : per;
+            chunks.push_back({static_cast<long long>(b0) * H, nb * H, nb, H, b0});
+        }
+    }
+    return chunks;
+}
+
+// Rounds of one launch: `units` units of equal cost on min(units, sms)
+// persistent CTAs, a short last round cut along the keys into parts when the
+// dense split applies (attn_launch's rule).
+double launch_rounds(long long units, int sms, int n_kv, bool dense)
+{
+    const long long G = units < sms ? units : sms;
+    const long long full = units / G, tail = units - full * G;
+    if (tail == 0)
+        return static_cast<double>(full);
+    long long parts = (dense && full >= 1) ? G / tail : 0;
+    if (parts > n_kv)
+        parts = n_kv;
+    return static_cast<double>(full) + (parts >= 2 ? 1.0 / static_cast<double>(parts) : 1.0);
+}
+
+// Cost model of the pipeline, used only to choose the chunk size: the host
+// link moves kLinkBps each way while both directions are busy (pinned
+// memory), a copy costs kCopyS more; a multiprocessor runs the kernel at
+// kSmFlops plus kUnitS per unit; a launch costs kLaunchS.
+constexpr double kLinkBps = 170e9;
+constexpr double kCopyS = 5e-6;
+constexpr double kSmFlops = 10.2e12;
+constexpr double kUnitS = 4e-6;
+constexpr double kLaunchS = 5e-6;
+
+// Modelled seconds of a call.  Chunk i's copy in follows chunk i-1's and the
+// kernel of the chunk that last held its slot; its kernel starts after its
+// copy in and that chunk's copy out, and -- the kernels of consecutive chunks
+// overlapping -- the GPU works through it as a fluid share of all
+// multiprocessors after the previous chunk, except that the last chunk's
+// short round is whole; its copy out follows chunk i-1's and its kernel.
+double model_seconds(const std::vector<HostChunk> &chunks, double in_row, double out_row, long long per_row,
+                     double unit_s, int sms, int n_kv, bool dense)
+{
+    const size_t n = chunks.size();
+    std::vector<double> up(n), gpu(n), down(n);
+    for (size_t i = 0; i < n; ++i) {
+        const double rows = chunks[i].rows;
+        const long long units = chunks[i].rows * per_row;
+        double t = i ? up[i - 1] : 0.0;
+        if (i >= kHostSlots && gpu[i - kHostSlots] > t)
+            t = gpu[i - kHostSlots];
+        up[i] = t + 3 * kCopyS + rows * in_row / kLinkBps;
+        double start = up[i];
+        if (i >= kHostSlots && down[i - kHostSlots] > start)
+            start = down[i - kHostSlots];
+        const double prev = i ? gpu[i - 1] : 0.0;
+        gpu[i] = (prev > start ? prev : start) + kLaunchS + static_cast<double>(units) * unit_s / sms;
+        if (i + 1 == n) {
+            const double whole = start + kLaunchS + launch_rounds(units, sms, n_kv, dense) * unit_s;
+            gpu[i] = whole > gpu[i] ? whole : gpu[i];
+        }
+        t = gpu[i];
+        if (i && down[i - 1] > t)
+            t = down[i - 1];
+        down[i] = t + 2 * kCopyS + rows * out_row / kLinkBps;
+    }
+    return n ? down[n - 1] : 0.0;
+}
+
+// Rows per chunk when the caller leaves it to the library: the candidate
+// with the shortest modelled call (at most 64 chunks; varlen: heads of one
+// sample or whole samples); fewer chunks on a tie.
+long long auto_chunk_rows(int B, int H, int Sq, int Skv, int D, const int *kv_lens, bool lse, int sms)
+{
+    const long long bh = static_cast<long long>(B) * H;
+    const bool varlen = kv_lens != nullptr;
+    const long long per_row = (static_cast<long long>(Sq) + 2 * vdx::BM - 1) / (2 * vdx::BM);
+    const int n_kv = (Skv + vdx::BN - 1) / vdx::BN;
+    double keys = static_cast<double>(n_kv) * vdx::BN;   // keys a unit visits (whole tiles)
+    if (varlen) {
+        double sum = 0.0;
+        for (int b = 0; b < B; ++b) {
+            const int L = kv_lens[b] < 0 ? 0 : (kv_lens[b] > Skv ? Skv : kv_lens[b]);
+            sum += static_cast<double>((L + vdx::BN - 1) / vdx::BN) * vdx::BN;
+        }
+        keys = B ? sum / B : 0.0;
+    }
+    const double unit_s = 2.0 * vdx::BM * keys * D * 4.0 / kSmFlops + kUnitS;
+    const double in_row = (static_cast<double>(Sq) + 2.0 * Skv) * D * 2.0;
+    const double out_row = static_cast<double>(Sq) * D * 2.0 + (lse ? 4.0 * Sq : 0.0);
+    std::vector<long long> cand;
+    if (!varlen) {
+        for (long long c = 1; c <= 64 && c <= bh; ++c)
+            cand.push_back((bh + c - 1) / c);
+    } else {
+        for (int c = 1; c <= H; ++c)
+            if (static_cast<long long>(B) * c <= 64)
+                cand.push_back((H + c - 1) / c);
+        for (int m = 2; m <= B; ++m)
+            if ((B + m - 1) / m <= 64)
+                cand.push_back(static_cast<long long>(m) * H);
+    }
+    long long best = bh;
+    double best_s = model_seconds(make_chunks(bh, B, H, varlen), in_row, out_row, per_row, unit_s, sms, n_kv, !varlen);
+    for (long long r : cand) {
+        const double t = model_seconds(make_chunks(r, B, H, varlen), in_row, out_row, per_row, unit_s, sms, n_kv,
+                                       !varlen);
+        if (t < best_s * 0.999 || (t <= best_s * 1.001 && r > best)) {
+            best_s = t;
+            best = r;
+        }
+    }
+    return best;
+}
+
 }  // namespace
 
 extern "C" {
@@ -448,6 +637,135 @@ int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, 
     rule.mode = vdx::MODE_VARLEN;
     rule.kv_lens = kv_lens;
     return attn_launch(q, k, v, out, lse, B, H, Sq, Skv_max, D, rule, scale, stream);
+}
+
+int vdx_attn_fwd_host(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,
+                      int Skv, int D, const int *kv_lens, float scale, long long chunk_rows, void *stream)
+{
+    // ---- validation (no CUDA calls)
+    if (!q || !k || !v || !out || B < 0 || H < 0 || Sq < 0 || Skv < 0 || (D != 64 && D != 128) ||
+        !std::isfinite(scale) || chunk_rows < 0)
+        return VDX_ERR_INVALID_ARG;
+    const long long bh = static_cast<long long>(B) * H;
+    if (bh == 0 || Sq == 0)
+        return VDX_OK;
+    if (bh > INT_MAX || static_cast<double>(bh) * (static_cast<double>(Sq) + Skv) * D > 1e17)
+        return VDX_ERR_INVALID_ARG;
+    const size_t row_q = static_cast<size_t>(Sq) * D * 2, row_kv = static_cast<size_t>(Skv) * D * 2;
+    const size_t row_l = static_cast<size_t>(Sq) * 4;
+    const size_t q_bytes = bh * row_q, kv_bytes = bh * row_kv, l_bytes = bh * row_l;
+    if (overlaps(out, q_bytes, q, q_bytes) ||
+        (kv_bytes && (overlaps(out, q_bytes, k, kv_bytes) || overlaps(out, q_bytes, v, kv_bytes))) ||
+        (lse && (overlaps(lse, l_bytes, out, q_bytes) || overlaps(lse, l_bytes, q, q_bytes) ||
+                 (kv_bytes && (overlaps(lse, l_bytes, k, kv_bytes) || overlaps(lse, l_bytes, v, kv_bytes))))))
+        return VDX_ERR_INVALID_ARG;
+    const bool varlen = kv_lens != nullptr;
+
+    // ---- device set-up
+    int sms = 0, dev = 0;
+    int st = device_ready(&sms);
+    if (st != VDX_OK)
+        return st;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return VDX_ERR_CUDA;
+
+    // ---- chunks
+    long long r = chunk_rows > 0 ? (chunk_rows < bh ? chunk_rows : bh)
+                                 : auto_chunk_rows(B, H, Sq, Skv, D, kv_lens, lse != nullptr, sms);
+    if (varlen && r > H)
+        r -= r % H;
+    const std::vector<HostChunk> chunks = make_chunks(r, B, H, varlen);
+    long long R = 0;
+    for (const HostChunk &c : chunks)
+        R = c.rows > R ? c.rows : R;
+
+    // ---- pipeline state and slots: [lens] then kHostSlots x [q | k | v | out | lse]
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    HostPipe &pp = host_pipe(dev, s);
+    std::lock_guard<std::mutex> lock(pp.mutex);
+    if ((st = host_pipe_init(pp)) != VDX_OK)
+        return st;
+    const size_t lens_b = round_up(static_cast<size_t>(B) * 4, 256);
+    const size_t sq_b = round_up(R * row_q, 256), skv_b = round_up(R * row_kv, 256);
+    const size_t sl_b = lse ? round_up(R * row_l, 256) : 0;
+    const size_t slot_b = 2 * sq_b + 2 * skv_b + sl_b;
+    if (pp.bytes < lens_b + kHostSlots * slot_b) {
+        if (pp.buf && cudaFree(pp.buf) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        pp.buf = nullptr;
+        pp.bytes = 0;
+        if (cudaMalloc(&pp.buf, lens_b + kHostSlots * slot_b) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        pp.bytes = lens_b + kHostSlots * slot_b;
+    }
+    char *base = static_cast<char *>(pp.buf);
+    int *d_lens = reinterpret_cast<int *>(base);
+    auto slot = [&](int i, int part) {   // part: 0 q, 1 k, 2 v, 3 out, 4 lse
+        const size_t off[5] = {0, sq_b, sq_b + skv_b, sq_b + 2 * skv_b, 2 * sq_b + 2 * skv_b};
+        return base + lens_b + static_cast<size_t>(i) * slot_b + off[part];
+    };
+
+    // ---- enqueue: everything after the caller's earlier work on `stream`
+    const char *qh = static_cast<const char *>(q), *kh = static_cast<const char *>(k);
+    const char *vh = static_cast<const char *>(v);
+    char *oh = static_cast<char *>(out), *lh = reinterpret_cast<char *>(lse);
+    if (cudaEventRecord(pp.start, s) != cudaSuccess || cudaStreamWaitEvent(pp.up, pp.start, 0) != cudaSuccess ||
+        cudaStreamWaitEvent(pp.run[0], pp.start, 0) != cudaSuccess ||
+        cudaStreamWaitEvent(pp.run[1], pp.start, 0) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    if (varlen && cudaMemcpyAsync(d_lens, kv_lens, static_cast<size_t>(B) * 4, cudaMemcpyHostToDevice, pp.up) !=
+                      cudaSuccess)
+        return VDX_ERR_CUDA;
+    const size_t n = chunks.size();
+    for (size_t i = 0; i <= n; ++i) {
+        if (i < n) {
+            // copy chunk i in once the slot's previous chunk has run, then run it
+            // once that chunk's results are out
+            const HostChunk &c = chunks[i];
+            const int sl = static_cast<int>(i % kHostSlots);
+            cudaStream_t rs = pp.run[i & 1];
+            if (i >= kHostSlots && cudaStreamWaitEvent(pp.up, pp.comp[sl], 0) != cudaSuccess)
+                return VDX_ERR_CUDA;
+            const size_t nq = c.rows * row_q, nkv = c.rows * row_kv;
+            if (cudaMemcpyAsync(slot(sl, 0), qh + c.row0 * row_q, nq, cudaMemcpyHostToDevice, pp.up) != cudaSuccess ||
+                (nkv && (cudaMemcpyAsync(slot(sl, 1), kh + c.row0 * row_kv, nkv, cudaMemcpyHostToDevice, pp.up) !=
+                             cudaSuccess ||
+                         cudaMemcpyAsync(slot(sl, 2), vh + c.row0 * row_kv, nkv, cudaMemcpyHostToDevice, pp.up) !=
+                             cudaSuccess)) ||
+                cudaEventRecord(pp.h2d[sl], pp.up) != cudaSuccess ||
+                cudaStreamWaitEvent(rs, pp.h2d[sl], 0) != cudaSuccess ||
+                (i >= kHostSlots && cudaStreamWaitEvent(rs, pp.d2h[sl], 0) != cudaSuccess))
+                return VDX_ERR_CUDA;
+            KeyRule rule;
+            if (varlen) {
+                rule.mode = vdx::MODE_VARLEN;
+                rule.kv_lens = d_lens + c.lens0;
+            }
+            st = attn_launch(slot(sl, 0), slot(sl, 1), slot(sl, 2), slot(sl, 3),
+                             lse ? reinterpret_cast<float *>(slot(sl, 4)) : nullptr, c.nb, c.nh, Sq, Skv, D, rule,
+                             scale, rs);
+            if (st != VDX_OK)
+                return st;
+            if (cudaEventRecord(pp.comp[sl], rs) != cudaSuccess)
+                return VDX_ERR_CUDA;
+        }
+        if (i >= 1) {
+            // copy chunk i-1 out once its kernel is done
+            const HostChunk &c = chunks[i - 1];
+            const int sl = static_cast<int>((i - 1) % kHostSlots);
+            if (cudaStreamWaitEvent(pp.down, pp.comp[sl], 0) != cudaSuccess ||
+                cudaMemcpyAsync(oh + c.row0 * row_q, slot(sl, 3), c.rows * row_q, cudaMemcpyDeviceToHost, pp.down) !=
+                    cudaSuccess ||
+                (lse && cudaMemcpyAsync(lh + c.row0 * row_l, slot(sl, 4), c.rows * row_l, cudaMemcpyDeviceToHost,
+                                        pp.down) != cudaSuccess) ||
+                cudaEventRecord(pp.d2h[sl], pp.down) != cudaSuccess)
+                return VDX_ERR_CUDA;
+        }
+    }
+    // the caller's stream resumes once the last result is on the host
+    if (cudaStreamWaitEvent(s, pp.d2h[(n - 1) % kHostSlots], 0) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    return VDX_OK;
 }
 
 int vdx_attn_fwd_win3d(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int F,

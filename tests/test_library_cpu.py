@@ -120,3 +120,35 @@ def test_binding_rejects_cpu_tensors():
     x = torch.zeros(1, 1, 4, 64, dtype=torch.bfloat16)
     with pytest.raises(TypeError):
         binding.attn_fwd(x, x, x)
+
+
+def test_host_entry_validation(lib):
+    """vdx_attn_fwd_host rejects bad arguments before any CUDA call."""
+    import torch
+    q = torch.zeros(1, 2, 8, 64, dtype=torch.bfloat16)
+    o = torch.zeros_like(q)
+    lse = torch.zeros(1, 2, 8)
+    a = (q.data_ptr(), q.data_ptr(), q.data_ptr())
+    f = lib.vdx_attn_fwd_host
+    assert f(None, *a[1:], o.data_ptr(), None, 1, 2, 8, 8, 64, None, 0.1, 0, None) == 1          # null q
+    assert f(*a, None, None, 1, 2, 8, 8, 64, None, 0.1, 0, None) == 1                            # null out
+    assert f(*a, o.data_ptr(), None, 1, 2, 8, 8, 96, None, 0.1, 0, None) == 1                    # bad D
+    assert f(*a, o.data_ptr(), None, 1, -2, 8, 8, 64, None, 0.1, 0, None) == 1                   # negative H
+    assert f(*a, o.data_ptr(), None, 1, 2, 8, 8, 64, None, 0.1, -1, None) == 1                   # chunk_rows < 0
+    assert f(*a, o.data_ptr(), None, 1, 2, 8, 8, 64, None, float("nan"), 0, None) == 1           # scale
+    assert f(*a, q.data_ptr(), None, 1, 2, 8, 8, 64, None, 0.1, 0, None) == 1                    # out aliases q
+    assert f(*a, o.data_ptr(), ctypes.cast(o.data_ptr(), ctypes.c_void_p), 1, 2, 8, 8, 64, None, 0.1, 0,
+             None) == 1                                                                          # lse inside out
+    assert f(*a, o.data_ptr(), lse.data_ptr(), 0, 2, 8, 8, 64, None, 0.1, 0, None) == 0          # no rows
+    assert f(*a, o.data_ptr(), lse.data_ptr(), 1, 2, 0, 8, 64, None, 0.1, 0, None) == 0          # no queries
+
+
+def test_binding_host_entry_rejects_cuda_layouts():
+    import torch
+    from paper_2609_18077_gb300 import binding
+    x = torch.zeros(1, 1, 4, 64, dtype=torch.float32)
+    with pytest.raises(TypeError):
+        binding.attn_fwd_host(x, x, x)
+    y = torch.zeros(1, 1, 4, 64, dtype=torch.bfloat16)
+    with pytest.raises(TypeError):
+        binding.attn_fwd_host(y, y, y, kv_lens=torch.zeros(2, dtype=torch.int32))
