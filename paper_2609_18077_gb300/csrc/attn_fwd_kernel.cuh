@@ -123,7 +123,7 @@ struct SegParams {
 
 // Shared-memory plan.  QBUF Q-tile pairs (2 = the next item's Q tiles load
 // while the current item runs) and NSTAGE K/V stages of (V_j, next K).
-template <int D, int QBUF, int NSTAGE_>
+template <int D, int QBUF, int NSTAGE_, bool OSTAGE = false>
 struct Layout {
     static_assert(D == 64 || D == 128, "head dim");
     static constexpr int TILE_BYTES = BM * D * 2;           // one Q, K or V tile
@@ -151,11 +151,28 @@ struct Layout {
     // [NSTAGE][4] listed modes: list entry of each stage's V tile; MODE_WIN also
     // the grid position of its first key (t | h << 16, w)
     static constexpr int ENTRY_OFF = (MERGE_OFF + 4 + 15) / 16 * 16;
-    // 197.8 KB in all configurations: under the 196 KB shared-memory carve-out
-    // (199,680 usable bytes), which leaves 60 KB of L1 for the spill slots.
-    static constexpr int BYTES = ENTRY_OFF + 16 * NSTAGE;
+    // OSTAGE: per softmax warp, a 32-row x 128-byte (64-column) box of O in the
+    // 128-byte swizzle of the output tensor map, written by the warp and stored
+    // by TMA.
+    static constexpr int OUT_BOX = 32 * 128;
+    static constexpr int OUT_OFF = (ENTRY_OFF + 16 * NSTAGE + 1023) / 1024 * 1024;
+    // Without OSTAGE 197.8 KB in all configurations: under the 196 KB
+    // shared-memory carve-out (199,680 usable bytes), which leaves 60 KB of L1
+    // for the spill slots.  With it 226 KB (the 228 KB carve-out).
+    static constexpr int BYTES = OSTAGE ? OUT_OFF + 8 * OUT_BOX : ENTRY_OFF + 16 * NSTAGE;
     static constexpr int ALLOC = BYTES + 1024;               // slack for 1024-B alignment
 };
+
+// O leaves through TMA stores from shared memory in the text cross-attention
+// instance, whose units are a few key tiles long: per-thread row stores (32
+// rows of one warp hit 32 cache lines per instruction) then keep the load-store
+// path busy long enough to delay the next unit's QK^T.  Elsewhere a unit runs
+// hundreds of key steps and the per-thread stores cost nothing measurable.
+template <int MODE>
+__host__ __device__ constexpr bool stages_out()
+{
+    return MODE == MODE_VARLEN;
+}
 
 __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, volatile int *abort_flag,
                                              uint64_t limit_ns)
@@ -466,10 +483,11 @@ __device__ __forceinline__ uint32_t tile_entry(const SegParams &sp, const Item &
 template <int D, int MODE, int QBUF, int NSTAGE>
 __global__ void __launch_bounds__(NUM_THREADS, 1)
     attn_fwd_kernel(const __grid_constant__ CUtensorMap tmap_q, const __grid_constant__ CUtensorMap tmap_k,
-                    const __grid_constant__ CUtensorMap tmap_v, const AttnParams p,
-                    const __grid_constant__ SegParams sp)
+                    const __grid_constant__ CUtensorMap tmap_v, const __grid_constant__ CUtensorMap tmap_o,
+                    const AttnParams p, const __grid_constant__ SegParams sp)
 {
-    using L = Layout<D, QBUF, NSTAGE>;
+    constexpr bool OSTAGE = stages_out<MODE>();
+    using L = Layout<D, QBUF, NSTAGE, OSTAGE>;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *sm = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     const uint32_t sbase = ptx::smem_u32(sm);
@@ -511,6 +529,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         ptx::tma_prefetch_desc(&tmap_q);
         ptx::tma_prefetch_desc(&tmap_k);
         ptx::tma_prefetch_desc(&tmap_v);
+        if (OSTAGE)
+            ptx::tma_prefetch_desc(&tmap_o);
     }
     ptx::tc_fence_before_sync();
     __syncthreads();
@@ -555,10 +575,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 // A padded sample's last V tile: rows past the valid length may
                 // hold any bits (NaN included) and 0 * NaN = NaN inside the
                 // GEMM, so stage the tile, zero those rows, then publish.
+                // The stage's K tile loads meanwhile: its bytes count on the
+                // full barrier, whose one arrival comes after the zeroing.
                 if (lane == 0) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_FIX), L::TILE_BYTES);
                     for (int h = 0; h < D / 64; ++h)
                         ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FIX), h * 64, vj * BN, vbh);
+                    if (has_k) {
+                        ptx::mbar_expect_tx(bar(L::B_FULL + st), L::TILE_BYTES);
+                        for (int h = 0; h < D / 64; ++h)
+                            ptx::tma_load_3d(kdst + h * L::HALF_BYTES, &tmap_k, bar(L::B_FULL + st), h * 64,
+                                             kj * BN, kbh);
+                    }
                 }
                 if (!__all_sync(0xffffffffu, wait_bounded(bar(L::B_FIX), fixes & 1, abort_flag, limit)))
                     return false;
@@ -575,7 +603,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 __syncwarp();
             }
             if (lane == 0) {
-                const uint32_t bytes = ((has_v && !fix) + has_k) * L::TILE_BYTES;
+                const uint32_t bytes = fix ? 0u : (has_v + has_k) * L::TILE_BYTES;
                 if (listed(MODE) && has_v) {
                     volatile uint32_t *slot = reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF) + 4 * st;
                     slot[0] = ventry;
@@ -967,7 +995,33 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 __syncwarp();
                 if (lane == 0)
                     ptx::mbar_arrive(bar(L::B_OE + t));
-                if (store) {
+                if (OSTAGE) {
+                    // This warp's 32 rows through its staging box, 64 columns at a
+                    // time: chunk c (16 bytes) of row r sits at chunk c ^ (r & 7).
+                    const uint32_t stg = sbase + L::OUT_OFF + (4 * t + wq) * L::OUT_BOX;
+                    const int row0 = (w.qp * 2 + t) * BM + wq * 32;
+#pragma unroll
+                    for (int h = 0; h < D / 64; ++h) {
+                        if (lane == 0)
+                            ptx::bulk_wait_read_all();   // the previous box was read out
+                        __syncwarp();
+#pragma unroll
+                        for (int c = 0; c < 8; ++c) {
+                            const uint32_t *src = &w16[2 * h + (c >> 2)][4 * (c & 3)];
+                            ptx::st_shared_v4(stg + lane * 128 + ((c ^ (lane & 7)) << 4), src[0], src[1], src[2],
+                                              src[3]);
+                        }
+                        ptx::fence_proxy_async_smem();
+                        __syncwarp();
+                        if (lane == 0 && row0 < p.Sq) {   // rows past Sq are clipped by the store
+                            ptx::tma_store_3d(&tmap_o, stg, h * 64, row0, w.bh);
+                            ptx::bulk_commit_group();
+                        }
+                    }
+                    if (store && p.lse)
+                        p.lse[static_cast<size_t>(w.bh) * p.Sq + q_row] =
+                            (m_used + __log2f(l_exact)) * 0.69314718055994530942f;
+                } else if (store) {
                     if (p.out_align32) {
                         // 32-byte stores: each fills a whole sector of the row.
 #pragma unroll
@@ -994,9 +1048,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             ++iq;
         }
         // An abort can leave this warp's tensor-memory loads or stores in
-        // flight; none may remain when the memory is released below.
+        // flight; none may remain when the memory is released below.  Nor may
+        // an output store still be reading its staging box.
         ptx::tmem_wait_ld();
         ptx::tmem_wait_st();
+        if (OSTAGE && lane == 0)
+            ptx::bulk_wait_all();
     }
 
     ptx::tc_fence_before_sync();

@@ -13,6 +13,7 @@
 #include <climits>
 #include <cmath>
 #include <cstdint>
+#include <cstring>
 #include <map>
 #include <mutex>
 #include <utility>
@@ -65,7 +66,7 @@ cudaError_t raise_smem_limit()
 {
     return cudaFuncSetAttribute(vdx::attn_fwd_kernel<D, MODE, QBUF, NSTAGE>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                vdx::Layout<D, QBUF, NSTAGE>::ALLOC);
+                                vdx::Layout<D, QBUF, NSTAGE, vdx::stages_out<MODE>()>::ALLOC);
 }
 
 cudaError_t raise_all_smem_limits()
@@ -83,10 +84,11 @@ cudaError_t raise_all_smem_limits()
 
 template <int D, int MODE, int QBUF, int NSTAGE>
 cudaError_t launch(dim3 grid, const CUtensorMap &mq, const CUtensorMap &mk, const CUtensorMap &mv,
-                   const vdx::AttnParams &p, const vdx::SegParams &sp, cudaStream_t s)
+                   const CUtensorMap &mo, const vdx::AttnParams &p, const vdx::SegParams &sp, cudaStream_t s)
 {
     vdx::attn_fwd_kernel<D, MODE, QBUF, NSTAGE>
-        <<<grid, vdx::NUM_THREADS, vdx::Layout<D, QBUF, NSTAGE>::ALLOC, s>>>(mq, mk, mv, p, sp);
+        <<<grid, vdx::NUM_THREADS, vdx::Layout<D, QBUF, NSTAGE, vdx::stages_out<MODE>()>::ALLOC, s>>>(mq, mk, mv, mo,
+                                                                                                      p, sp);
     return cudaGetLastError();
 }
 
@@ -157,13 +159,13 @@ int workspace(int dev, cudaStream_t stream, size_t bytes, void **out)
 
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-// [B*H, rows, D] bf16 tensor as a 3-D TMA map with 64 x 128 x 1 boxes, 128-B swizzle.
-int make_map(CUtensorMap *map, const void *base, long long rows, long long bh, int D)
+// [B*H, rows, D] bf16 tensor as a 3-D TMA map with 64 x box_rows x 1 boxes, 128-B swizzle.
+int make_map(CUtensorMap *map, const void *base, long long rows, long long bh, int D, int box_rows = vdx::BM)
 {
     const cuuint64_t dims[3] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(rows),
                                 static_cast<cuuint64_t>(bh)};
     const cuuint64_t strides[2] = {static_cast<cuuint64_t>(D) * 2, static_cast<cuuint64_t>(rows) * D * 2};
-    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(vdx::BM), 1};
+    const cuuint32_t box[3] = {64, static_cast<cuuint32_t>(box_rows), 1};
     const cuuint32_t estr[3] = {1, 1, 1};
     const CUresult r = encode_fn()(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides,
                                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -232,10 +234,15 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     if (st != VDX_OK)
         return st;
 
-    CUtensorMap mq, mk, mv;
+    CUtensorMap mq, mk, mv, mo;
     const long long kv_rows = Skv > 0 ? Skv : 1;   // never loaded when Skv == 0
     if ((st = make_map(&mq, q, Sq, bh, D)) != VDX_OK || (st = make_map(&mk, k, kv_rows, bh, D)) != VDX_OK ||
         (st = make_map(&mv, v, kv_rows, bh, D)) != VDX_OK)
+        return st;
+    // The output map (32-row boxes, one per softmax warp) serves the instance
+    // that stores O through TMA; the others never read it.
+    std::memset(&mo, 0, sizeof(mo));
+    if (varlen && (st = make_map(&mo, out, Sq, bh, D, 32)) != VDX_OK)
         return st;
 
     vdx::AttnParams p{};
@@ -359,15 +366,15 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     using vdx::MODE_WIN;
     cudaError_t e;
     if (D == 128) {
-        e = varlen ? launch<128, MODE_VARLEN, 1, 2>(grid, mq, mk, mv, p, sp, s)
-                   : seg ? launch<128, MODE_SEG, 1, 2>(grid, mq, mk, mv, p, sp, s)
-                         : win ? launch<128, MODE_WIN, 1, 2>(grid, mq, mk, mv, p, sp, s)
-                               : launch<128, MODE_DENSE, 1, 2>(grid, mq, mk, mv, p, sp, s);
+        e = varlen ? launch<128, MODE_VARLEN, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
+                   : seg ? launch<128, MODE_SEG, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
+                         : win ? launch<128, MODE_WIN, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
+                               : launch<128, MODE_DENSE, 1, 2>(grid, mq, mk, mv, mo, p, sp, s);
     } else {
-        e = varlen ? launch<64, MODE_VARLEN, 2, 4>(grid, mq, mk, mv, p, sp, s)
-                   : seg ? launch<64, MODE_SEG, 2, 4>(grid, mq, mk, mv, p, sp, s)
-                         : win ? launch<64, MODE_WIN, 2, 4>(grid, mq, mk, mv, p, sp, s)
-                               : launch<64, MODE_DENSE, 2, 4>(grid, mq, mk, mv, p, sp, s);
+        e = varlen ? launch<64, MODE_VARLEN, 2, 4>(grid, mq, mk, mv, mo, p, sp, s)
+                   : seg ? launch<64, MODE_SEG, 2, 4>(grid, mq, mk, mv, mo, p, sp, s)
+                         : win ? launch<64, MODE_WIN, 2, 4>(grid, mq, mk, mv, mo, p, sp, s)
+                               : launch<64, MODE_DENSE, 2, 4>(grid, mq, mk, mv, mo, p, sp, s);
     }
     if (e == cudaErrorNoKernelImageForDevice)
         return VDX_ERR_DEVICE;
