@@ -17,9 +17,10 @@ max over ranks is reported.  Inputs (Q, K, V, O: 403 MB) exceed the 129 MB
 L2, so no flush is inserted.  SM clocks are sampled with nvidia-smi during
 the timed region.  A second timed pass ("e2e") starts from pinned host
 buffers: every step copies Q, K, V host->device, runs the kernel and copies
-O and LSE back.  Dense and padded-text steps are one vdx_attn_fwd_host call
-(the library cuts the (b, h) rows into chunks and overlaps the copies with
-the kernel); the other workloads copy, run the step and copy back in turn.
+O and LSE back.  Each step is one host-buffer call (vdx_attn_fwd_host, or its
+segment or window variant: the library cuts the (b, h) rows into chunks and
+overlaps the copies with the kernel); the RoPE workload copies, runs its
+three kernels and copies back in turn.
 
 --impl reference times the fp64 CPU oracle (the only reference this
 method has) on a bounded row sample of the same workload.  Under torchrun
@@ -249,13 +250,20 @@ def run_ours(args):
         (0 if sh is None else sum(t.numel() * 4 for t in sh))
     d2h = oh.numel() * oh.element_size() + lseh.numel() * lseh.element_size()
 
-    host_api = segs is None and wl.window is None and wl.rope is None
+    host_api = wl.rope is None
 
     def e2e_step():
         if host_api:
-            # one vdx_attn_fwd_host call: chunked, copies overlapped with the kernel
-            binding.attn_fwd_host(qh, kh, vh, kv_lens=lh, scale=wl.scale, out=oh, lse=lseh, device=dev,
-                                  synchronize=False)
+            # one host-buffer call: chunked, copies overlapped with the kernel
+            if wl.window is not None:
+                binding.attn_fwd_win3d_host(qh, kh, vh, wl.latent, wl.window[0], wl.window[1], scale=wl.scale,
+                                            out=oh, lse=lseh, device=dev, synchronize=False)
+            elif sh is not None:
+                binding.attn_fwd_segments_host(qh, kh, vh, sh[0], sh[1], scale=wl.scale, out=oh, lse=lseh,
+                                               device=dev, synchronize=False)
+            else:
+                binding.attn_fwd_host(qh, kh, vh, kv_lens=lh, scale=wl.scale, out=oh, lse=lseh, device=dev,
+                                      synchronize=False)
             return
         q.copy_(qh, non_blocking=True)
         k.copy_(kh, non_blocking=True)
@@ -309,8 +317,10 @@ def run_ours(args):
         "clocks": clocks,
         "e2e": {"value": round(e2e_tflops, 2), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "path": ("vdx_attn_fwd_host: pinned host buffers, chunks of (b, h) rows, copies in and out "
-                         "overlapped with the kernel" if host_api else
+                "path": ("host-buffer entry point (vdx_attn_fwd%s_host): pinned host buffers, chunks of (b, h) "
+                         "rows, copies in and out overlapped with the kernel" % (
+                             "_win3d" if wl.window is not None else ("_segments" if sh is not None else ""))
+                         if host_api else
                          "pinned host buffers copied in, the step's kernels, results copied out")},
         "gpu_launches": args.steps * launches_per_step,
         "roofline": {"bound": "tensor", "achieved": round(per_launch_tflops, 2), "peak": peak,

@@ -206,6 +206,26 @@ int vdx_attn_fwd_host(const void *q, const void *k, const void *v, void *out, fl
                       int B, int H, int Sq, int Skv, int D, const int *kv_lens, float scale,
                       long long chunk_rows, void *stream);
 
+/*
+ * vdx_attn_fwd_segments on HOST buffers, through the same pipeline as
+ * vdx_attn_fwd_host.  q_seg [B, Sq] and kv_seg [B, Skv] are HOST int32
+ * arrays, copied in once per call; chunks hold heads of one sample or whole
+ * samples.  Results and errors as vdx_attn_fwd_segments; memory as
+ * vdx_attn_fwd_host plus B*(Sq+Skv) ints for the ids.
+ */
+int vdx_attn_fwd_segments_host(const void *q, const void *k, const void *v, void *out, float *lse,
+                               int B, int H, int Sq, int Skv, int D, const int *q_seg, const int *kv_seg,
+                               float scale, long long chunk_rows, void *stream);
+
+/*
+ * vdx_attn_fwd_win3d on HOST buffers, through the same pipeline as
+ * vdx_attn_fwd_host (every (b, h) shares the grid, so a chunk is any block of
+ * rows).  Results and errors as vdx_attn_fwd_win3d.
+ */
+int vdx_attn_fwd_win3d_host(const void *q, const void *k, const void *v, void *out, float *lse,
+                            int B, int H, int F, int Hp, int Wp, int D, int kt, int kh, int kw,
+                            int neighbourhood, float scale, long long chunk_rows, void *stream);
+
 /* Human-readable name of a vdx_status (static storage; never NULL). */
 const char *vdx_status_string(int status);
 

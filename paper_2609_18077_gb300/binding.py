@@ -36,6 +36,9 @@ SIGNATURES = {
     "vdx_attn_fwd_win3d": (_I, [_P, _P, _P, _P, _P] + [_I] * 10 + [ctypes.c_float, _P]),
     "vdx_rope3d": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _I, _I, _I, ctypes.c_float, _I, _P]),
     "vdx_attn_fwd_host": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, ctypes.c_float, ctypes.c_longlong, _P]),
+    "vdx_attn_fwd_segments_host": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, ctypes.c_float,
+                                        ctypes.c_longlong, _P]),
+    "vdx_attn_fwd_win3d_host": (_I, [_P, _P, _P, _P, _P] + [_I] * 10 + [ctypes.c_float, ctypes.c_longlong, _P]),
     "vdx_status_string": (ctypes.c_char_p, [_I]),
     "vdx_check_device_error": (_I, [_P]),
     "vdx_selftest_wait_timeout": (_I, [_I, _P]),
@@ -235,6 +238,49 @@ def attn_fwd_win3d(q, k, v, grid, window, neighbourhood=True, scale=None, out=No
     return out, lse
 
 
+def _host_check(q, k, v):
+    """Checks CPU q, k, v."""
+    for name, t in (("q", q), ("k", k), ("v", v)):
+        if not isinstance(t, torch.Tensor) or t.device.type != "cpu":
+            raise TypeError(f"{name} must be a CPU tensor")
+        if t.dtype != torch.bfloat16 or t.dim() != 4 or not t.is_contiguous():
+            raise TypeError(f"{name} must be a contiguous bf16 [B,H,S,D] tensor")
+    if k.shape != v.shape or q.shape[:2] != k.shape[:2] or q.shape[3] != k.shape[3]:
+        raise ValueError(f"shape mismatch q{tuple(q.shape)} k{tuple(k.shape)} v{tuple(v.shape)}")
+
+
+def _host_outputs(q, out, lse, return_lse):
+    """Makes (or checks) the CPU outputs: pinned when made here."""
+    B, H, Sq, D = q.shape
+    if out is None:
+        out = torch.empty(q.shape, dtype=torch.bfloat16, pin_memory=True)
+    elif (out.device.type != "cpu" or out.shape != q.shape or out.dtype != torch.bfloat16
+          or not out.is_contiguous()):
+        raise ValueError("out must be a contiguous bf16 CPU tensor shaped like q")
+    if lse is None and return_lse:
+        lse = torch.empty((B, H, Sq), dtype=torch.float32, pin_memory=True)
+    elif lse is not None and (lse.device.type != "cpu" or lse.shape != (B, H, Sq)
+                              or lse.dtype != torch.float32 or not lse.is_contiguous()):
+        raise ValueError("lse must be a contiguous fp32 [B,H,Sq] CPU tensor")
+    return out, lse
+
+
+def _host_ints(x, shape, name):
+    if (not isinstance(x, torch.Tensor) or x.device.type != "cpu" or x.dtype != torch.int32
+            or tuple(x.shape) != tuple(shape) or not x.is_contiguous()):
+        raise TypeError(f"{name} must be a contiguous int32 CPU tensor of shape {list(shape)}")
+
+
+def _host_call(fn, name, args, device, synchronize):
+    device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    with torch.cuda.device(device):
+        st = fn(*args, _stream_handle(device))
+        if st != VDX_OK:
+            raise VdxError(st, name)
+        if synchronize:
+            torch.cuda.current_stream(device).synchronize()
+
+
 def attn_fwd_host(q, k, v, kv_lens=None, scale=None, out=None, lse=None, return_lse=True, chunk_rows=0,
                   device=None, synchronize=True):
     """Attention forward on host tensors through ``vdx_attn_fwd_host``.
@@ -247,38 +293,52 @@ def attn_fwd_host(q, k, v, kv_lens=None, scale=None, out=None, lse=None, return_
     synchronize=False the results are complete only once that stream is
     synchronised.  Returns (out, lse or None).
     """
-    for name, t in (("q", q), ("k", k), ("v", v)):
-        if not isinstance(t, torch.Tensor) or t.device.type != "cpu":
-            raise TypeError(f"{name} must be a CPU tensor")
-        if t.dtype != torch.bfloat16 or t.dim() != 4 or not t.is_contiguous():
-            raise TypeError(f"{name} must be a contiguous bf16 [B,H,S,D] tensor")
-    if k.shape != v.shape or q.shape[:2] != k.shape[:2] or q.shape[3] != k.shape[3]:
-        raise ValueError(f"shape mismatch q{tuple(q.shape)} k{tuple(k.shape)} v{tuple(v.shape)}")
+    _host_check(q, k, v)
+    B, H, Sq, D = q.shape
+    if kv_lens is not None:
+        _host_ints(kv_lens, (B,), "kv_lens")
+    out, lse = _host_outputs(q, out, lse, return_lse)
+    scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
+    _host_call(load().vdx_attn_fwd_host, "vdx_attn_fwd_host",
+               (q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                lse.data_ptr() if lse is not None else None, B, H, Sq, k.shape[2], D,
+                kv_lens.data_ptr() if kv_lens is not None else None, scale, int(chunk_rows)), device, synchronize)
+    return out, lse
+
+
+def attn_fwd_segments_host(q, k, v, q_seg, kv_seg, scale=None, out=None, lse=None, return_lse=True, chunk_rows=0,
+                           device=None, synchronize=True):
+    """Joint attention with segment ids on host tensors through
+    ``vdx_attn_fwd_segments_host``; q_seg int32 [B, Sq], kv_seg int32 [B, Skv]
+    (CPU).  Other arguments as attn_fwd_host."""
+    _host_check(q, k, v)
     B, H, Sq, D = q.shape
     Skv = k.shape[2]
-    if kv_lens is not None and (not isinstance(kv_lens, torch.Tensor) or kv_lens.device.type != "cpu"
-                                or kv_lens.dtype != torch.int32 or kv_lens.shape != (B,)
-                                or not kv_lens.is_contiguous()):
-        raise TypeError("kv_lens must be a contiguous int32 CPU tensor of shape [B]")
-    if out is None:
-        out = torch.empty(q.shape, dtype=torch.bfloat16, pin_memory=True)
-    elif (out.device.type != "cpu" or out.shape != q.shape or out.dtype != torch.bfloat16
-          or not out.is_contiguous()):
-        raise ValueError("out must be a contiguous bf16 CPU tensor shaped like q")
-    if lse is None and return_lse:
-        lse = torch.empty((B, H, Sq), dtype=torch.float32, pin_memory=True)
-    elif lse is not None and (lse.device.type != "cpu" or lse.shape != (B, H, Sq)
-                              or lse.dtype != torch.float32 or not lse.is_contiguous()):
-        raise ValueError("lse must be a contiguous fp32 [B,H,Sq] CPU tensor")
+    _host_ints(q_seg, (B, Sq), "q_seg")
+    _host_ints(kv_seg, (B, Skv), "kv_seg")
+    out, lse = _host_outputs(q, out, lse, return_lse)
     scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
-    device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
-    with torch.cuda.device(device):
-        st = load().vdx_attn_fwd_host(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
-                                      lse.data_ptr() if lse is not None else None, B, H, Sq, Skv, D,
-                                      kv_lens.data_ptr() if kv_lens is not None else None, scale,
-                                      int(chunk_rows), _stream_handle(device))
-        if st != VDX_OK:
-            raise VdxError(st, "vdx_attn_fwd_host")
-        if synchronize:
-            torch.cuda.current_stream(device).synchronize()
+    _host_call(load().vdx_attn_fwd_segments_host, "vdx_attn_fwd_segments_host",
+               (q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                lse.data_ptr() if lse is not None else None, B, H, Sq, Skv, D, q_seg.data_ptr(),
+                kv_seg.data_ptr(), scale, int(chunk_rows)), device, synchronize)
+    return out, lse
+
+
+def attn_fwd_win3d_host(q, k, v, grid, window, neighbourhood=True, scale=None, out=None, lse=None,
+                        return_lse=True, chunk_rows=0, device=None, synchronize=True):
+    """Windowed 3D attention on host tensors through ``vdx_attn_fwd_win3d_host``;
+    grid = (F, Hp, Wp), window = (kt, kh, kw) as attn_fwd_win3d.  Other
+    arguments as attn_fwd_host."""
+    _host_check(q, k, v)
+    B, H, S, D = q.shape
+    F, Hp, Wp = (int(x) for x in grid)
+    if S != F * Hp * Wp or k.shape[2] != S:
+        raise ValueError(f"q, k, v must hold the F*Hp*Wp = {F * Hp * Wp} grid tokens")
+    out, lse = _host_outputs(q, out, lse, return_lse)
+    scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
+    _host_call(load().vdx_attn_fwd_win3d_host, "vdx_attn_fwd_win3d_host",
+               (q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                lse.data_ptr() if lse is not None else None, B, H, F, Hp, Wp, D, int(window[0]), int(window[1]),
+                int(window[2]), int(bool(neighbourhood)), scale, int(chunk_rows)), device, synchronize)
     return out, lse

@@ -420,6 +420,26 @@ int noalloc_scratch(void **ptr)
     return st.status;
 }
 
+// Window rule of vdx_attn_fwd_win3d(_host): odd window sizes >= 1, grid sides
+// below 65536 (window bounds are packed in 16 bits), F*Hp*Wp within int.
+int win_rule(int F, int Hp, int Wp, int kt, int kh, int kw, int neighbourhood, KeyRule *rule)
+{
+    if (F < 0 || Hp < 0 || Wp < 0 || kt < 1 || kh < 1 || kw < 1 || !(kt & kh & kw & 1))
+        return VDX_ERR_INVALID_ARG;
+    const long long S = static_cast<long long>(F) * Hp * Wp;
+    if (S > INT_MAX || F > 65535 || Hp > 65535 || Wp > 65535)
+        return VDX_ERR_UNSUPPORTED;
+    rule->mode = vdx::MODE_WIN;
+    rule->win.F = F;
+    rule->win.Hp = Hp;
+    rule->win.Wp = Wp;
+    rule->win.kt = kt;
+    rule->win.kh = kh;
+    rule->win.kw = kw;
+    rule->win.neighbourhood = neighbourhood ? 1 : 0;
+    return VDX_OK;
+}
+
 // ---------------------------------------------------------------- host-buffer pipeline
 // vdx_attn_fwd_host cuts the (b, h) rows into chunks.  Chunk i is copied in
 // on one stream, run on one of two compute streams (alternating, so that
@@ -468,20 +488,22 @@ int host_pipe_init(HostPipe &pp)
 }
 
 // A chunk: rows [row0, row0 + rows) of the flattened (b, h) rows, launched as
-// B x H = nb x nh; its valid key counts start at kv_lens[lens0].
+// B x H = nb x nh; its per-sample data (text lengths, segment ids) starts at
+// sample b0.
 struct HostChunk {
     long long row0;
     int rows, nb, nh;
-    long long lens0;
+    long long b0;
 };
 
-// Chunks of r rows; varlen chunks hold heads of one sample (r <= H) or whole
-// samples (r a multiple of H), so that one kv_lens offset serves a launch.
-std::vector<HostChunk> make_chunks(long long r, int B, int H, bool varlen)
+// Chunks of r rows.  With per-sample data a chunk holds heads of one sample
+// (r <= H) or whole samples (r a multiple of H), so that one offset into that
+// data serves a launch.
+std::vector<HostChunk> make_chunks(long long r, int B, int H, bool per_sample)
 {
     std::vector<HostChunk> chunks;
     const long long bh = static_cast<long long>(B) * H;
-    if (!varlen) {
+    if (!per_sample) {
         for (long long r0 = 0; r0 < bh; r0 += r) {
             const int n = static_cast<int>(bh - r0 < r ? bh - r0 : r);
             chunks.push_back({r0, n, 1, n, 0});
@@ -563,16 +585,19 @@ double model_seconds(const std::vector<HostChunk> &chunks, double in_row, double
 }
 
 // Rows per chunk when the caller leaves it to the library: the candidate
-// with the shortest modelled call (at most 64 chunks; varlen: heads of one
-// sample or whole samples); fewer chunks on a tie.
-long long auto_chunk_rows(int B, int H, int Sq, int Skv, int D, const int *kv_lens, bool lse, int sms)
+// with the shortest modelled call (at most 64 chunks; with per-sample data,
+// heads of one sample or whole samples); fewer chunks on a tie.  kv_lens
+// (host, may be NULL) refines the keys a unit visits; otherwise every key
+// tile counts (an upper bound for segment and window problems).
+long long auto_chunk_rows(int B, int H, int Sq, int Skv, int D, const int *kv_lens, bool per_sample, bool lse,
+                          int sms)
 {
     const long long bh = static_cast<long long>(B) * H;
-    const bool varlen = kv_lens != nullptr;
+    const bool varlen = per_sample;
     const long long per_row = (static_cast<long long>(Sq) + 2 * vdx::BM - 1) / (2 * vdx::BM);
     const int n_kv = (Skv + vdx::BN - 1) / vdx::BN;
     double keys = static_cast<double>(n_kv) * vdx::BN;   // keys a unit visits (whole tiles)
-    if (varlen) {
+    if (kv_lens) {
         double sum = 0.0;
         for (int b = 0; b < B; ++b) {
             const int L = kv_lens[b] < 0 ? 0 : (kv_lens[b] > Skv ? Skv : kv_lens[b]);
@@ -606,6 +631,151 @@ long long auto_chunk_rows(int B, int H, int Sq, int Skv, int D, const int *kv_le
         }
     }
     return best;
+}
+
+// The host-buffer pipeline behind vdx_attn_fwd_host and its segment and
+// window variants.  hr holds HOST pointers to the per-sample data (kv_lens
+// [B]; q_seg [B, Sq] and kv_seg [B, Skv]); they are copied to the device once
+// per call.  Window problems share one grid, so their chunks are any rows.
+int host_pipeline(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
+                  int D, const KeyRule &hr, float scale, long long chunk_rows, void *stream)
+{
+    // ---- validation (no CUDA calls)
+    const bool varlen = hr.mode == vdx::MODE_VARLEN, seg = hr.mode == vdx::MODE_SEG;
+    if (!q || !k || !v || !out || B < 0 || H < 0 || Sq < 0 || Skv < 0 || (D != 64 && D != 128) ||
+        !std::isfinite(scale) || chunk_rows < 0 || (varlen && !hr.kv_lens) || (seg && (!hr.q_seg || !hr.kv_seg)))
+        return VDX_ERR_INVALID_ARG;
+    const long long bh = static_cast<long long>(B) * H;
+    if (bh == 0 || Sq == 0)
+        return VDX_OK;
+    if (bh > INT_MAX || static_cast<double>(bh) * (static_cast<double>(Sq) + Skv) * D > 1e17)
+        return VDX_ERR_INVALID_ARG;
+    const size_t row_q = static_cast<size_t>(Sq) * D * 2, row_kv = static_cast<size_t>(Skv) * D * 2;
+    const size_t row_l = static_cast<size_t>(Sq) * 4;
+    const size_t q_bytes = bh * row_q, kv_bytes = bh * row_kv, l_bytes = bh * row_l;
+    if (overlaps(out, q_bytes, q, q_bytes) ||
+        (kv_bytes && (overlaps(out, q_bytes, k, kv_bytes) || overlaps(out, q_bytes, v, kv_bytes))) ||
+        (lse && (overlaps(lse, l_bytes, out, q_bytes) || overlaps(lse, l_bytes, q, q_bytes) ||
+                 (kv_bytes && (overlaps(lse, l_bytes, k, kv_bytes) || overlaps(lse, l_bytes, v, kv_bytes))))))
+        return VDX_ERR_INVALID_ARG;
+    const bool per_sample = varlen || seg;
+
+    // ---- device set-up
+    int sms = 0, dev = 0;
+    int st = device_ready(&sms);
+    if (st != VDX_OK)
+        return st;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return VDX_ERR_CUDA;
+
+    // ---- chunks
+    long long r = chunk_rows > 0 ? (chunk_rows < bh ? chunk_rows : bh)
+                                 : auto_chunk_rows(B, H, Sq, Skv, D, hr.kv_lens, per_sample, lse != nullptr, sms);
+    if (per_sample && r > H)
+        r -= r % H;
+    const std::vector<HostChunk> chunks = make_chunks(r, B, H, per_sample);
+    long long R = 0;
+    for (const HostChunk &c : chunks)
+        R = c.rows > R ? c.rows : R;
+
+    // ---- pipeline state and slots: [per-sample data] then kHostSlots x [q | k | v | out | lse]
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    HostPipe &pp = host_pipe(dev, s);
+    std::lock_guard<std::mutex> lock(pp.mutex);
+    if ((st = host_pipe_init(pp)) != VDX_OK)
+        return st;
+    const size_t qseg_b = seg ? round_up(static_cast<size_t>(B) * Sq * 4, 256) : 0;
+    const size_t lens_b = varlen ? round_up(static_cast<size_t>(B) * 4, 256)
+                                 : (seg ? qseg_b + round_up(static_cast<size_t>(B) * Skv * 4, 256) : 0);
+    const size_t sq_b = round_up(R * row_q, 256), skv_b = round_up(R * row_kv, 256);
+    const size_t sl_b = lse ? round_up(R * row_l, 256) : 0;
+    const size_t slot_b = 2 * sq_b + 2 * skv_b + sl_b;
+    if (pp.bytes < lens_b + kHostSlots * slot_b) {
+        if (pp.buf && cudaFree(pp.buf) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        pp.buf = nullptr;
+        pp.bytes = 0;
+        if (cudaMalloc(&pp.buf, lens_b + kHostSlots * slot_b) != cudaSuccess)
+            return VDX_ERR_CUDA;
+        pp.bytes = lens_b + kHostSlots * slot_b;
+    }
+    char *base = static_cast<char *>(pp.buf);
+    int *d_lens = reinterpret_cast<int *>(base);                 // varlen: [B]
+    int *d_qseg = reinterpret_cast<int *>(base);                 // segments: [B, Sq], then [B, Skv]
+    int *d_kvseg = reinterpret_cast<int *>(base + qseg_b);
+    auto slot = [&](int i, int part) {   // part: 0 q, 1 k, 2 v, 3 out, 4 lse
+        const size_t off[5] = {0, sq_b, sq_b + skv_b, sq_b + 2 * skv_b, 2 * sq_b + 2 * skv_b};
+        return base + lens_b + static_cast<size_t>(i) * slot_b + off[part];
+    };
+
+    // ---- enqueue: everything after the caller's earlier work on `stream`
+    const char *qh = static_cast<const char *>(q), *kh = static_cast<const char *>(k);
+    const char *vh = static_cast<const char *>(v);
+    char *oh = static_cast<char *>(out), *lh = reinterpret_cast<char *>(lse);
+    if (cudaEventRecord(pp.start, s) != cudaSuccess || cudaStreamWaitEvent(pp.up, pp.start, 0) != cudaSuccess ||
+        cudaStreamWaitEvent(pp.run[0], pp.start, 0) != cudaSuccess ||
+        cudaStreamWaitEvent(pp.run[1], pp.start, 0) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    if (varlen && cudaMemcpyAsync(d_lens, hr.kv_lens, static_cast<size_t>(B) * 4, cudaMemcpyHostToDevice, pp.up) !=
+                      cudaSuccess)
+        return VDX_ERR_CUDA;
+    if (seg && (cudaMemcpyAsync(d_qseg, hr.q_seg, static_cast<size_t>(B) * Sq * 4, cudaMemcpyHostToDevice, pp.up) !=
+                    cudaSuccess ||
+                (Skv > 0 && cudaMemcpyAsync(d_kvseg, hr.kv_seg, static_cast<size_t>(B) * Skv * 4,
+                                            cudaMemcpyHostToDevice, pp.up) != cudaSuccess)))
+        return VDX_ERR_CUDA;
+    const size_t n = chunks.size();
+    for (size_t i = 0; i <= n; ++i) {
+        if (i < n) {
+            // copy chunk i in once the slot's previous chunk has run, then run it
+            // once that chunk's results are out
+            const HostChunk &c = chunks[i];
+            const int sl = static_cast<int>(i % kHostSlots);
+            cudaStream_t rs = pp.run[i & 1];
+            if (i >= kHostSlots && cudaStreamWaitEvent(pp.up, pp.comp[sl], 0) != cudaSuccess)
+                return VDX_ERR_CUDA;
+            const size_t nq = c.rows * row_q, nkv = c.rows * row_kv;
+            if (cudaMemcpyAsync(slot(sl, 0), qh + c.row0 * row_q, nq, cudaMemcpyHostToDevice, pp.up) != cudaSuccess ||
+                (nkv && (cudaMemcpyAsync(slot(sl, 1), kh + c.row0 * row_kv, nkv, cudaMemcpyHostToDevice, pp.up) !=
+                             cudaSuccess ||
+                         cudaMemcpyAsync(slot(sl, 2), vh + c.row0 * row_kv, nkv, cudaMemcpyHostToDevice, pp.up) !=
+                             cudaSuccess)) ||
+                cudaEventRecord(pp.h2d[sl], pp.up) != cudaSuccess ||
+                cudaStreamWaitEvent(rs, pp.h2d[sl], 0) != cudaSuccess ||
+                (i >= kHostSlots && cudaStreamWaitEvent(rs, pp.d2h[sl], 0) != cudaSuccess))
+                return VDX_ERR_CUDA;
+            KeyRule rule = hr;   // window problems: the grid as given
+            if (varlen)
+                rule.kv_lens = d_lens + c.b0;
+            if (seg) {
+                rule.q_seg = d_qseg + c.b0 * Sq;
+                rule.kv_seg = d_kvseg + c.b0 * Skv;
+            }
+            st = attn_launch(slot(sl, 0), slot(sl, 1), slot(sl, 2), slot(sl, 3),
+                             lse ? reinterpret_cast<float *>(slot(sl, 4)) : nullptr, c.nb, c.nh, Sq, Skv, D, rule,
+                             scale, rs);
+            if (st != VDX_OK)
+                return st;
+            if (cudaEventRecord(pp.comp[sl], rs) != cudaSuccess)
+                return VDX_ERR_CUDA;
+        }
+        if (i >= 1) {
+            // copy chunk i-1 out once its kernel is done
+            const HostChunk &c = chunks[i - 1];
+            const int sl = static_cast<int>((i - 1) % kHostSlots);
+            if (cudaStreamWaitEvent(pp.down, pp.comp[sl], 0) != cudaSuccess ||
+                cudaMemcpyAsync(oh + c.row0 * row_q, slot(sl, 3), c.rows * row_q, cudaMemcpyDeviceToHost, pp.down) !=
+                    cudaSuccess ||
+                (lse && cudaMemcpyAsync(lh + c.row0 * row_l, slot(sl, 4), c.rows * row_l, cudaMemcpyDeviceToHost,
+                                        pp.down) != cudaSuccess) ||
+                cudaEventRecord(pp.d2h[sl], pp.down) != cudaSuccess)
+                return VDX_ERR_CUDA;
+        }
+    }
+    // the caller's stream resumes once the last result is on the host
+    if (cudaStreamWaitEvent(s, pp.d2h[(n - 1) % kHostSlots], 0) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    return VDX_OK;
 }
 
 }  // namespace
@@ -649,150 +819,47 @@ int vdx_attn_fwd_varlen(const void *q, const void *k, const void *v, void *out, 
 int vdx_attn_fwd_host(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,
                       int Skv, int D, const int *kv_lens, float scale, long long chunk_rows, void *stream)
 {
-    // ---- validation (no CUDA calls)
-    if (!q || !k || !v || !out || B < 0 || H < 0 || Sq < 0 || Skv < 0 || (D != 64 && D != 128) ||
-        !std::isfinite(scale) || chunk_rows < 0)
-        return VDX_ERR_INVALID_ARG;
-    const long long bh = static_cast<long long>(B) * H;
-    if (bh == 0 || Sq == 0)
-        return VDX_OK;
-    if (bh > INT_MAX || static_cast<double>(bh) * (static_cast<double>(Sq) + Skv) * D > 1e17)
-        return VDX_ERR_INVALID_ARG;
-    const size_t row_q = static_cast<size_t>(Sq) * D * 2, row_kv = static_cast<size_t>(Skv) * D * 2;
-    const size_t row_l = static_cast<size_t>(Sq) * 4;
-    const size_t q_bytes = bh * row_q, kv_bytes = bh * row_kv, l_bytes = bh * row_l;
-    if (overlaps(out, q_bytes, q, q_bytes) ||
-        (kv_bytes && (overlaps(out, q_bytes, k, kv_bytes) || overlaps(out, q_bytes, v, kv_bytes))) ||
-        (lse && (overlaps(lse, l_bytes, out, q_bytes) || overlaps(lse, l_bytes, q, q_bytes) ||
-                 (kv_bytes && (overlaps(lse, l_bytes, k, kv_bytes) || overlaps(lse, l_bytes, v, kv_bytes))))))
-        return VDX_ERR_INVALID_ARG;
-    const bool varlen = kv_lens != nullptr;
+    KeyRule rule;
+    if (kv_lens) {
+        rule.mode = vdx::MODE_VARLEN;
+        rule.kv_lens = kv_lens;
+    }
+    return host_pipeline(q, k, v, out, lse, B, H, Sq, Skv, D, rule, scale, chunk_rows, stream);
+}
 
-    // ---- device set-up
-    int sms = 0, dev = 0;
-    int st = device_ready(&sms);
+int vdx_attn_fwd_segments_host(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H,
+                               int Sq, int Skv, int D, const int *q_seg, const int *kv_seg, float scale,
+                               long long chunk_rows, void *stream)
+{
+    KeyRule rule;
+    rule.mode = vdx::MODE_SEG;
+    rule.q_seg = q_seg;
+    rule.kv_seg = kv_seg;
+    return host_pipeline(q, k, v, out, lse, B, H, Sq, Skv, D, rule, scale, chunk_rows, stream);
+}
+
+int vdx_attn_fwd_win3d_host(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int F,
+                            int Hp, int Wp, int D, int kt, int kh, int kw, int neighbourhood, float scale,
+                            long long chunk_rows, void *stream)
+{
+    KeyRule rule;
+    const int st = win_rule(F, Hp, Wp, kt, kh, kw, neighbourhood, &rule);
     if (st != VDX_OK)
         return st;
-    if (cudaGetDevice(&dev) != cudaSuccess)
-        return VDX_ERR_CUDA;
-
-    // ---- chunks
-    long long r = chunk_rows > 0 ? (chunk_rows < bh ? chunk_rows : bh)
-                                 : auto_chunk_rows(B, H, Sq, Skv, D, kv_lens, lse != nullptr, sms);
-    if (varlen && r > H)
-        r -= r % H;
-    const std::vector<HostChunk> chunks = make_chunks(r, B, H, varlen);
-    long long R = 0;
-    for (const HostChunk &c : chunks)
-        R = c.rows > R ? c.rows : R;
-
-    // ---- pipeline state and slots: [lens] then kHostSlots x [q | k | v | out | lse]
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
-    HostPipe &pp = host_pipe(dev, s);
-    std::lock_guard<std::mutex> lock(pp.mutex);
-    if ((st = host_pipe_init(pp)) != VDX_OK)
-        return st;
-    const size_t lens_b = round_up(static_cast<size_t>(B) * 4, 256);
-    const size_t sq_b = round_up(R * row_q, 256), skv_b = round_up(R * row_kv, 256);
-    const size_t sl_b = lse ? round_up(R * row_l, 256) : 0;
-    const size_t slot_b = 2 * sq_b + 2 * skv_b + sl_b;
-    if (pp.bytes < lens_b + kHostSlots * slot_b) {
-        if (pp.buf && cudaFree(pp.buf) != cudaSuccess)
-            return VDX_ERR_CUDA;
-        pp.buf = nullptr;
-        pp.bytes = 0;
-        if (cudaMalloc(&pp.buf, lens_b + kHostSlots * slot_b) != cudaSuccess)
-            return VDX_ERR_CUDA;
-        pp.bytes = lens_b + kHostSlots * slot_b;
-    }
-    char *base = static_cast<char *>(pp.buf);
-    int *d_lens = reinterpret_cast<int *>(base);
-    auto slot = [&](int i, int part) {   // part: 0 q, 1 k, 2 v, 3 out, 4 lse
-        const size_t off[5] = {0, sq_b, sq_b + skv_b, sq_b + 2 * skv_b, 2 * sq_b + 2 * skv_b};
-        return base + lens_b + static_cast<size_t>(i) * slot_b + off[part];
-    };
-
-    // ---- enqueue: everything after the caller's earlier work on `stream`
-    const char *qh = static_cast<const char *>(q), *kh = static_cast<const char *>(k);
-    const char *vh = static_cast<const char *>(v);
-    char *oh = static_cast<char *>(out), *lh = reinterpret_cast<char *>(lse);
-    if (cudaEventRecord(pp.start, s) != cudaSuccess || cudaStreamWaitEvent(pp.up, pp.start, 0) != cudaSuccess ||
-        cudaStreamWaitEvent(pp.run[0], pp.start, 0) != cudaSuccess ||
-        cudaStreamWaitEvent(pp.run[1], pp.start, 0) != cudaSuccess)
-        return VDX_ERR_CUDA;
-    if (varlen && cudaMemcpyAsync(d_lens, kv_lens, static_cast<size_t>(B) * 4, cudaMemcpyHostToDevice, pp.up) !=
-                      cudaSuccess)
-        return VDX_ERR_CUDA;
-    const size_t n = chunks.size();
-    for (size_t i = 0; i <= n; ++i) {
-        if (i < n) {
-            // copy chunk i in once the slot's previous chunk has run, then run it
-            // once that chunk's results are out
-            const HostChunk &c = chunks[i];
-            const int sl = static_cast<int>(i % kHostSlots);
-            cudaStream_t rs = pp.run[i & 1];
-            if (i >= kHostSlots && cudaStreamWaitEvent(pp.up, pp.comp[sl], 0) != cudaSuccess)
-                return VDX_ERR_CUDA;
-            const size_t nq = c.rows * row_q, nkv = c.rows * row_kv;
-            if (cudaMemcpyAsync(slot(sl, 0), qh + c.row0 * row_q, nq, cudaMemcpyHostToDevice, pp.up) != cudaSuccess ||
-                (nkv && (cudaMemcpyAsync(slot(sl, 1), kh + c.row0 * row_kv, nkv, cudaMemcpyHostToDevice, pp.up) !=
-                             cudaSuccess ||
-                         cudaMemcpyAsync(slot(sl, 2), vh + c.row0 * row_kv, nkv, cudaMemcpyHostToDevice, pp.up) !=
-                             cudaSuccess)) ||
-                cudaEventRecord(pp.h2d[sl], pp.up) != cudaSuccess ||
-                cudaStreamWaitEvent(rs, pp.h2d[sl], 0) != cudaSuccess ||
-                (i >= kHostSlots && cudaStreamWaitEvent(rs, pp.d2h[sl], 0) != cudaSuccess))
-                return VDX_ERR_CUDA;
-            KeyRule rule;
-            if (varlen) {
-                rule.mode = vdx::MODE_VARLEN;
-                rule.kv_lens = d_lens + c.lens0;
-            }
-            st = attn_launch(slot(sl, 0), slot(sl, 1), slot(sl, 2), slot(sl, 3),
-                             lse ? reinterpret_cast<float *>(slot(sl, 4)) : nullptr, c.nb, c.nh, Sq, Skv, D, rule,
-                             scale, rs);
-            if (st != VDX_OK)
-                return st;
-            if (cudaEventRecord(pp.comp[sl], rs) != cudaSuccess)
-                return VDX_ERR_CUDA;
-        }
-        if (i >= 1) {
-            // copy chunk i-1 out once its kernel is done
-            const HostChunk &c = chunks[i - 1];
-            const int sl = static_cast<int>((i - 1) % kHostSlots);
-            if (cudaStreamWaitEvent(pp.down, pp.comp[sl], 0) != cudaSuccess ||
-                cudaMemcpyAsync(oh + c.row0 * row_q, slot(sl, 3), c.rows * row_q, cudaMemcpyDeviceToHost, pp.down) !=
-                    cudaSuccess ||
-                (lse && cudaMemcpyAsync(lh + c.row0 * row_l, slot(sl, 4), c.rows * row_l, cudaMemcpyDeviceToHost,
-                                        pp.down) != cudaSuccess) ||
-                cudaEventRecord(pp.d2h[sl], pp.down) != cudaSuccess)
-                return VDX_ERR_CUDA;
-        }
-    }
-    // the caller's stream resumes once the last result is on the host
-    if (cudaStreamWaitEvent(s, pp.d2h[(n - 1) % kHostSlots], 0) != cudaSuccess)
-        return VDX_ERR_CUDA;
-    return VDX_OK;
+    const int S = F * Hp * Wp;
+    return host_pipeline(q, k, v, out, lse, B, H, S, S, D, rule, scale, chunk_rows, stream);
 }
+
 
 int vdx_attn_fwd_win3d(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int F,
                        int Hp, int Wp, int D, int kt, int kh, int kw, int neighbourhood, float scale, void *stream)
 {
-    if (F < 0 || Hp < 0 || Wp < 0 || kt < 1 || kh < 1 || kw < 1 || !(kt & kh & kw & 1))
-        return VDX_ERR_INVALID_ARG;
-    const long long S = static_cast<long long>(F) * Hp * Wp;
-    if (S > INT_MAX || F > 65535 || Hp > 65535 || Wp > 65535)   // window bounds are packed in 16 bits
-        return VDX_ERR_UNSUPPORTED;
     KeyRule rule;
-    rule.mode = vdx::MODE_WIN;
-    rule.win.F = F;
-    rule.win.Hp = Hp;
-    rule.win.Wp = Wp;
-    rule.win.kt = kt;
-    rule.win.kh = kh;
-    rule.win.kw = kw;
-    rule.win.neighbourhood = neighbourhood ? 1 : 0;
-    return attn_launch(q, k, v, out, lse, B, H, static_cast<int>(S), static_cast<int>(S), D, rule, scale, stream);
+    const int st = win_rule(F, Hp, Wp, kt, kh, kw, neighbourhood, &rule);
+    if (st != VDX_OK)
+        return st;
+    const int S = F * Hp * Wp;
+    return attn_launch(q, k, v, out, lse, B, H, S, S, D, rule, scale, stream);
 }
 
 int vdx_rope3d(const void *x, void *y, int B, int H, int S, int D, int F, int Hp, int Wp, int s0, int d_t, int d_h,

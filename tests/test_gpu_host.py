@@ -125,3 +125,39 @@ def test_workload_host_path(name):
                                                scale=w["scale"])
         assert torch.equal(out, o_dev.cpu()) and torch.equal(lse, l_dev.cpu())
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("r", [0, 1, 2, 4, 6])
+def test_segments_host_bit_identical_to_one_device_call(r):
+    """Joint text-video ids (padded text slots in their own segment); chunks of
+    heads of one sample (r <= H) or of whole samples (r = 4 rounds down to 3)."""
+    from paper_2609_18077_gb300 import binding, workloads
+    B, H, S, D = 2, 3, 700, 64
+    seg = workloads.joint_segments([37, 120], 130, S)
+    q, k, v = workloads.random_qkv(B, H, S, S, D, 4500 + r, 2.0)
+    scale = D ** -0.5
+    qs = torch.from_numpy(seg)
+    out, lse = binding.attn_fwd_segments_host(*(t.pin_memory() for t in (q, k, v)), qs, qs, scale=scale,
+                                              chunk_rows=r)
+    o_dev, l_dev = binding.attn_fwd_segments(q.cuda(), k.cuda(), v.cuda(), qs.cuda(), qs.cuda(), scale=scale)
+    assert torch.equal(out, o_dev.cpu())
+    assert torch.equal(lse, l_dev.cpu())
+    o_ref, lse_ref = run_oracle(q, k, v, scale, q_seg=seg, kv_seg=seg)
+    compare(out, lse, o_ref, lse_ref)
+
+
+@pytest.mark.parametrize("r", [0, 1, 5])
+def test_win3d_host_bit_identical_to_one_device_call(r):
+    from paper_2609_18077_gb300 import binding, workloads
+    B, H, D = 1, 5, 128
+    grid, window = (4, 6, 20), (3, 3, 5)
+    S = grid[0] * grid[1] * grid[2]
+    q, k, v = workloads.random_qkv(B, H, S, S, D, 4600 + r, 2.0)
+    scale = D ** -0.5
+    out, lse = binding.attn_fwd_win3d_host(*(t.pin_memory() for t in (q, k, v)), grid, window, True, scale=scale,
+                                           chunk_rows=r)
+    o_dev, l_dev = binding.attn_fwd_win3d(q.cuda(), k.cuda(), v.cuda(), grid, window, True, scale=scale)
+    assert torch.equal(out, o_dev.cpu())
+    assert torch.equal(lse, l_dev.cpu())
+    o_ref, lse_ref = run_oracle(q, k, v, scale, window=(grid, window, True))
+    compare(out, lse, o_ref, lse_ref)

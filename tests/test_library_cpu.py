@@ -152,3 +152,25 @@ def test_binding_host_entry_rejects_cuda_layouts():
     y = torch.zeros(1, 1, 4, 64, dtype=torch.bfloat16)
     with pytest.raises(TypeError):
         binding.attn_fwd_host(y, y, y, kv_lens=torch.zeros(2, dtype=torch.int32))
+
+
+def test_segment_and_window_host_entries_validate(lib):
+    """The segment and window host entries reject bad arguments before any CUDA call."""
+    import torch
+    q = torch.zeros(1, 2, 8, 64, dtype=torch.bfloat16)
+    o = torch.zeros_like(q)
+    ids = torch.zeros(1, 8, dtype=torch.int32)
+    a = (q.data_ptr(), q.data_ptr(), q.data_ptr(), o.data_ptr(), None)
+    f = lib.vdx_attn_fwd_segments_host
+    assert f(*a, 1, 2, 8, 8, 64, None, ids.data_ptr(), 0.1, 0, None) == 1                  # no q_seg
+    assert f(*a, 1, 2, 8, 8, 64, ids.data_ptr(), None, 0.1, 0, None) == 1                  # no kv_seg
+    assert f(*a, 1, 2, 8, 8, 64, ids.data_ptr(), ids.data_ptr(), 0.1, -3, None) == 1       # chunk_rows
+    assert f(*a, 0, 2, 8, 8, 64, ids.data_ptr(), ids.data_ptr(), 0.1, 0, None) == 0        # no rows
+    g = lib.vdx_attn_fwd_win3d_host
+    assert g(*a, 1, 2, 2, 2, 2, 64, 2, 3, 3, 1, 0.1, 0, None) == 1                        # even window
+    assert g(*a, 1, 2, 70000, 1, 1, 64, 3, 3, 3, 1, 0.1, 0, None) == 2                    # grid side
+    assert g(*a, 1, 2, 2, 2, 2, 96, 3, 3, 3, 1, 0.1, 0, None) == 1                        # bad D
+    assert g(*a, 1, 2, 0, 2, 2, 64, 3, 3, 3, 1, 0.1, 0, None) == 0                        # no tokens
+    from paper_2609_18077_gb300 import binding
+    with pytest.raises(TypeError):
+        binding.attn_fwd_segments_host(q, q, q, ids, torch.zeros(1, 7, dtype=torch.int32))
