@@ -121,6 +121,11 @@ WORKLOADS = {
         "large720", B=1, H=40, D=128, Sq=75600, Skv=75600, seed=1005, latent=(21, 45, 80),
         oracle_rows=4096,
         description="large-DiT 720p self-attention, latent 21x45x80 -> 75600 tokens"),
+    "large720_h4": Workload(
+        "large720_h4", B=1, H=4, D=128, Sq=75600, Skv=75600, seed=1005, latent=(21, 45, 80),
+        oracle_rows=4096,
+        description="large720's sequence with 4 heads: the same kernel and unit length at a tenth of the "
+                    "device memory, for multi-pass profiler captures"),
     "rope480": Workload(
         "rope480", B=1, H=12, D=128, Sq=32760, Skv=32760, seed=1002, latent=(21, 30, 52),
         logit_gain=math.sqrt(3.0), oracle_rows=4096,
