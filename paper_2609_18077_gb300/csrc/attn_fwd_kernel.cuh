@@ -646,22 +646,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const Item w = item_at<MODE>(p, sp, cta, i);
             const int ni = next_with_keys(i);
             const int qb = iq % QBUF;
-            if (iq >= QBUF) {
-                // Q buffer qb is free once its previous item's last QK^T ran.
-                const int ph = ((iq / QBUF) - 1) & 1;
-                ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_QE + 2 * qb), ph, abort_flag, limit) &&
-                                                 wait_bounded(bar(L::B_QE + 2 * qb + 1), ph, abort_flag, limit));
-                if (!ok)
-                    break;
-            }
-            if (lane == 0) {
-                for (int t = 0; t < 2; ++t) {
+            // Each Q tile of buffer qb is free once its previous item's last
+            // QK^T ran; tile 0's load starts without waiting for tile 1's.
+            for (int t = 0; ok && t < 2; ++t) {
+                if (iq >= QBUF)
+                    ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_QE + 2 * qb + t), ((iq / QBUF) - 1) & 1,
+                                                              abort_flag, limit));
+                if (ok && lane == 0) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_Q + 2 * qb + t), L::TILE_BYTES);
                     for (int h = 0; h < D / 64; ++h)
                         ptx::tma_load_3d(sbase + L::Q_OFF + (2 * qb + t) * L::TILE_BYTES + h * L::HALF_BYTES,
                                          &tmap_q, bar(L::B_Q + 2 * qb + t), h * 64, (w.qp * 2 + t) * BM, w.bh);
                 }
             }
+            if (!ok)
+                break;
             Item nw;
             nw.ok = false;
             if (ni >= 0)
@@ -710,8 +709,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     ok = wait_bounded(bar(L::B_FULL + 0), 0, abort_flag, limit);   // first key tile
                 const int qb = iq % QBUF;
                 const int qph = (iq / QBUF) & 1;
-                ok = ok && wait_bounded(bar(L::B_Q + 2 * qb), qph, abort_flag, limit) &&
-                     wait_bounded(bar(L::B_Q + 2 * qb + 1), qph, abort_flag, limit);
+                // Each tile's first QK^T as soon as that tile's Q landed.
+                ok = ok && wait_bounded(bar(L::B_Q + 2 * qb), qph, abort_flag, limit);
                 if (!ok)
                     break;
                 const uint64_t dq0 = dq_base + (2 * qb) * TILE16;
@@ -721,6 +720,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 ptx::tc_fence_after_sync();
                 issue_qk<D>(s0, dq0, dk + st_k0 * STAGE16);
                 ptx::mma_commit(bar(L::B_S + 0));
+                if (!(ok = wait_bounded(bar(L::B_Q + 2 * qb + 1), qph, abort_flag, limit)))
+                    break;
+                ptx::tc_fence_after_sync();
                 issue_qk<D>(s1, dq1, dk + st_k0 * STAGE16);
                 ptx::mma_commit(bar(L::B_S + 1));
                 // That stage also carried the previous item's last V: both are done now.
