@@ -181,7 +181,7 @@ int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out,
  * host memory.  The library copies the inputs in, runs the kernel and copies
  * the results out, overlapping the three: the (b, h) rows are cut into
  * chunks, and chunk i's kernel runs while chunk i+1 is copied in and chunk
- * i-1 copied out, on two copy streams of the library's own.
+ * i-1 copied out.
  *   q, k, v, out, lse, kv_lens : HOST pointers, caller-owned, laid out as in
  *          vdx_attn_fwd(_varlen) (kv_lens: int32 [B], read by the host during
  *          the call and copied in); lse may be NULL.  No alignment rule.  out
@@ -196,11 +196,17 @@ int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out,
  * the host buffers are pinned (page-locked); pageable buffers give the same
  * results with the copies serialised by the CUDA runtime.  The host buffers
  * must stay valid until `stream` is synchronised.
- * Memory: per (device, stream), two device slots of one chunk's q, k, v, out
- * and lse each (~270 MB for B=1, H=12, S=32760, D=128 at the default
- * chunking), allocated by the first call, grown by a larger one (which waits
- * for the device), kept until the process exits; plus vdx_attn_fwd's
- * workspace.  Errors: as vdx_attn_fwd; chunk_rows < 0 is VDX_ERR_INVALID_ARG.
+ * Streams: besides `stream`, the library's own copy-in and copy-out streams
+ * and two compute streams that alternate over the chunks (so that a chunk's
+ * kernel fills the multiprocessors the previous one's last round leaves
+ * idle).  Each chunk's kernel is vdx_attn_fwd(_varlen) on those rows, so the
+ * results are bit for bit those of such calls.
+ * Memory: per (device, stream), three device slots of one chunk's q, k, v,
+ * out and lse each (~100 MB for B=1, H=12, S=32760, D=128 at the default
+ * chunking of one row), allocated by the first call, grown by a larger one
+ * (which waits for the device), kept until the process exits; plus
+ * vdx_attn_fwd's workspace per compute stream.  Errors: as vdx_attn_fwd;
+ * chunk_rows < 0 is VDX_ERR_INVALID_ARG.
  */
 int vdx_attn_fwd_host(const void *q, const void *k, const void *v, void *out, float *lse,
                       int B, int H, int Sq, int Skv, int D, const int *kv_lens, float scale,

@@ -5,8 +5,9 @@
 // then three 3-D TMA tensor maps (head dim, sequence, batch*head) are encoded
 // and one kernel is launched on the caller's stream (joint attention with
 // segment ids first launches two small kernels that build its key-tile
-// lists).  The only allocation is the workspace of the split tail and of the
-// key-tile lists (per device and stream, made once, grown, kept).
+// lists).  The device calls allocate only the workspace of the split tail and
+// of the key-tile lists (per device and stream, made once, grown, kept); the
+// host-buffer calls also keep their pipeline's staging slots and streams.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
