@@ -76,3 +76,34 @@ def test_noalloc_matches_allocating_entry_point(lib, B, H, Sq, Skv, D):
     assert free_after == free_before, "vdx_attn_fwd_noalloc changed free device memory"
     for g, r in zip(got, refs):
         _close(g, r)
+
+
+@pytest.mark.parametrize("B,H,Sq,Skv,D", SHAPES)
+def test_noalloc_in_cuda_graph(lib, B, H, Sq, Skv, D):
+    """Captured into a CUDA graph (the call allocates nothing, so capture is
+    legal) and replayed on new inputs copied into the captured buffers: every
+    replay matches an eager vdx_attn_fwd call on the same inputs."""
+    from paper_2609_18077_gb300 import binding, workloads
+    scale = 1.0 / math.sqrt(D)
+    q, k, v = (t.cuda() for t in workloads.random_qkv(B, H, Sq, Skv, D, seed=950, logit_gain=1.6))
+    outputs = _outputs(q)
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        _run(lib.vdx_attn_fwd_noalloc, q, k, v, scale, outputs)   # first call: looks up the scratch
+    torch.cuda.current_stream().wait_stream(side)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=side):
+        _run(lib.vdx_attn_fwd_noalloc, q, k, v, scale, outputs)
+    for s in range(3):
+        nq, nk, nv = (t.cuda() for t in workloads.random_qkv(B, H, Sq, Skv, D, seed=960 + s, logit_gain=1.6))
+        q.copy_(nq)
+        k.copy_(nk)
+        v.copy_(nv)
+        graph.replay()
+        torch.cuda.synchronize()
+        assert binding.check_device_error() == binding.VDX_OK
+        ref = _run(lib.vdx_attn_fwd, nq, nk, nv, scale, _outputs(nq))
+        torch.cuda.synchronize()
+        _close(outputs, ref)
