@@ -3,8 +3,8 @@
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
 
 One step = one attention forward (one vdx_attn_fwd / vdx_attn_fwd_varlen /
-vdx_attn_fwd_segments / vdx_attn_fwd_win3d call, preceded by two
-vdx_rope3d calls for the rope workload) over the whole workload, inputs
+vdx_attn_fwd_segments / vdx_attn_fwd_win3d / vdx_attn_fwd_rope3d call) over
+the whole workload, inputs
 resident in HBM.  The default workload is the small-DiT 480p self-attention (B=1, H=12,
 D=128, S = 21*30*52 = 32760 tokens, logit std ~3).  FLOPs = 4*B*H*Sq*Skv*D
 (effective key counts for the padded-text workload; the (query, key) pairs
@@ -166,18 +166,17 @@ def run_ours(args):
         launches_per_step = 2     # key-tile lists, then the attention
     rope = wl.rope
     if rope is not None:
-        # the step rotates Q and K into buffers of their own, then attends
-        q_r, k_r = torch.empty_like(q), torch.empty_like(k)
+        # the step turns Q and K (two RoPE launches), then attends
+        q_r = torch.empty_like(q)   # the standalone RoPE timing's output
         launches_per_step = 3
 
     def step():
         if wl.window is not None:
             binding.attn_fwd_win3d(q, k, v, wl.latent, wl.window[0], wl.window[1], scale=wl.scale, out=out, lse=lse)
         elif rope is not None:
+            # one call: Q and K turned into the library's buffers, then the attention
             grid, s0, dims, theta, inter = rope
-            binding.rope3d(q, grid, s0, dims, theta, inter, out=q_r)
-            binding.rope3d(k, grid, s0, dims, theta, inter, out=k_r)
-            binding.attn_fwd(q_r, k_r, v, scale=wl.scale, out=out, lse=lse)
+            binding.attn_fwd_rope3d(q, k, v, grid, s0, dims, theta, inter, scale=wl.scale, out=out, lse=lse)
         elif segs is not None:
             binding.attn_fwd_segments(q, k, v, segs[0], segs[1], scale=wl.scale, out=out, lse=lse)
         elif lens is None:

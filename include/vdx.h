@@ -148,6 +148,25 @@ int vdx_rope3d(const void *x, void *y, int B, int H, int S, int D, int F, int Hp
                int d_t, int d_h, int d_w, float theta, int interleaved, void *stream);
 
 /*
+ * Self-attention with the 3D rotary embedding applied to q and k (Sec. 2:
+ * each family's 3D RoPE before its flash attention): exactly
+ *   vdx_rope3d(q -> q'), vdx_rope3d(k -> k'), vdx_attn_fwd(q', k', v)
+ * with Sq = Skv = S and the RoPE arguments of vdx_rope3d, so the results are
+ * bit for bit those of these three calls; q and k are not modified.  q' and
+ * k' live in two library buffers of B*H*S*D bf16 each per (device, stream),
+ * allocated by the first call, grown when needed, kept until exit; plus
+ * vdx_attn_fwd's workspace.  (K cannot be turned inside the attention: every
+ * query unit of a head reads all of K.  Turning each Q tile in shared memory
+ * after it lands was measured 0.9 % slower per call than the separate pass.)
+ * Arguments and errors as vdx_rope3d and vdx_attn_fwd together (D 64 or 128;
+ * q, k, v, out 16-byte aligned).
+ */
+int vdx_attn_fwd_rope3d(const void *q, const void *k, const void *v, void *out, float *lse,
+                        int B, int H, int S, int D, int F, int Hp, int Wp, int s0,
+                        int d_t, int d_h, int d_w, float theta, int interleaved,
+                        float scale, void *stream);
+
+/*
  * vdx_attn_fwd without any device allocation (the paper has no counterpart;
  * this is a library service).  Same arguments, results and errors as
  * vdx_attn_fwd, for callers that must not allocate device memory: code that

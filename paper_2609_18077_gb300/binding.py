@@ -35,6 +35,7 @@ SIGNATURES = {
     "vdx_attn_fwd_noalloc": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, ctypes.c_float, _P]),
     "vdx_attn_fwd_win3d": (_I, [_P, _P, _P, _P, _P] + [_I] * 10 + [ctypes.c_float, _P]),
     "vdx_rope3d": (_I, [_P, _P, _I, _I, _I, _I, _I, _I, _I, _I, _I, _I, _I, ctypes.c_float, _I, _P]),
+    "vdx_attn_fwd_rope3d": (_I, [_P, _P, _P, _P, _P] + [_I] * 11 + [ctypes.c_float, _I, ctypes.c_float, _P]),
     "vdx_attn_fwd_host": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, ctypes.c_float, ctypes.c_longlong, _P]),
     "vdx_attn_fwd_segments_host": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, ctypes.c_float,
                                         ctypes.c_longlong, _P]),
@@ -213,6 +214,32 @@ def rope3d(x, grid, s0, dims, theta, interleaved=True, out=None):
     if st != VDX_OK:
         raise VdxError(st, "vdx_rope3d")
     return out
+
+
+def attn_fwd_rope3d(q, k, v, grid, s0, dims, theta, interleaved=True, scale=None, out=None, lse=None,
+                    return_lse=True):
+    """Self-attention with the 3D RoPE of q and k, through ``vdx_attn_fwd_rope3d``:
+    bit for bit rope3d(q), rope3d(k), then attn_fwd, with the turned tensors in
+    library buffers; q and k unchanged.
+
+    q, k, v: bf16 [B,H,S,D] (CUDA); grid = (F, Hp, Wp); dims = (d_t, d_h, d_w).
+    """
+    _check_qkv(q, k, v)
+    B, H, S, D = q.shape
+    if k.shape[2] != S:
+        raise ValueError("q and k must hold the same tokens")
+    F, Hp, Wp = (int(x) for x in grid)
+    d_t, d_h, d_w = (int(x) for x in dims)
+    scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
+    out, lse = _outputs(q, out, lse, return_lse)
+    with torch.cuda.device(q.device):
+        st = load().vdx_attn_fwd_rope3d(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                                        lse.data_ptr() if lse is not None else None, B, H, S, D, F, Hp, Wp,
+                                        int(s0), d_t, d_h, d_w, float(theta), int(bool(interleaved)), scale,
+                                        _stream_handle(q.device))
+    if st != VDX_OK:
+        raise VdxError(st, "vdx_attn_fwd_rope3d")
+    return out, lse
 
 
 def attn_fwd_win3d(q, k, v, grid, window, neighbourhood=True, scale=None, out=None, lse=None, return_lse=True):

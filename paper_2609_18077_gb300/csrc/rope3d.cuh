@@ -35,6 +35,48 @@ struct RopeParams {
     int copy_all;           // y != x: also write the untouched pairs and tokens
 };
 
+// Axis part of rotated pair `pair` (< (d_t + d_h + d_w) / 2): its axis a
+// (0 t, 1 h, 2 w), its index i inside the part, the part's width da and first
+// dim base.
+__device__ __forceinline__ void pair_axis(const RopeParams &p, int pair, int &a, int &i, int &da, int &base)
+{
+    a = 0;
+    base = 0;
+    da = p.d_t;
+    i = pair;
+    if (i >= p.d_t / 2) {
+        i -= p.d_t / 2;
+        base = p.d_t;
+        da = p.d_h;
+        a = 1;
+        if (i >= p.d_h / 2) {
+            i -= p.d_h / 2;
+            base += p.d_h;
+            da = p.d_w;
+            a = 2;
+        }
+    }
+}
+
+// theta^(-2i/da) as 2^(-2i/da * log2 theta).
+__device__ __forceinline__ float pair_inv_freq(int i, int da, float log2_theta)
+{
+    return exp2f(-2.f * static_cast<float>(i) / static_cast<float>(da) * log2_theta);
+}
+
+// Cosine and sine of pos * inv_freq.  The angle is reduced to [-pi, pi]
+// (Cody and Waite: 2 pi = 6.28125, exact in few bits, plus a small
+// remainder, so k * 6.28125 is exact), then the fast sine and cosine, whose
+// documented error on that interval is 2^-21.4.
+__device__ __forceinline__ void turn_angle(int pos, float inv_freq, float &c, float &sn)
+{
+    float ph = static_cast<float>(pos) * inv_freq;
+    const float k = rintf(ph * 0.15915494309189535f);
+    ph = fmaf(-k, 6.28125f, ph);
+    ph = fmaf(-k, 1.9353071795864769253e-3f, ph);
+    __sincosf(ph, &sn, &c);
+}
+
 // Pair `pair` of a row: its two element indices, and whether and how far it turns
 // for grid offset g (g outside [0, F*Hp*Wp): no turn).
 template <bool INTER>
@@ -50,20 +92,8 @@ __device__ __forceinline__ bool pair_turn(const RopeParams &p, int pair, long lo
         ib = ia + 1;
         return false;
     }
-    // axis part of this pair and its index i inside the part
-    int a = 0, base = 0, da = p.d_t, i = pair;
-    if (i >= p.d_t / 2) {
-        i -= p.d_t / 2;
-        base = p.d_t;
-        da = p.d_h;
-        a = 1;
-        if (i >= p.d_h / 2) {
-            i -= p.d_h / 2;
-            base += p.d_h;
-            da = p.d_w;
-            a = 2;
-        }
-    }
+    int a, i, da, base;
+    pair_axis(p, pair, a, i, da, base);
     ia = base + (INTER ? 2 * i : i);
     ib = base + (INTER ? 2 * i + 1 : i + da / 2);
     if (!on_grid)
@@ -71,16 +101,20 @@ __device__ __forceinline__ bool pair_turn(const RopeParams &p, int pair, long lo
     const long long hw = static_cast<long long>(p.Hp) * p.Wp;
     const int pos = a == 0 ? static_cast<int>(g / hw)
                            : (a == 1 ? static_cast<int>((g / p.Wp) % p.Hp) : static_cast<int>(g % p.Wp));
-    const float inv_freq = exp2f(-2.f * static_cast<float>(i) / static_cast<float>(da) * p.log2_theta);
-    // Reduce the angle to [-pi, pi] (Cody and Waite: 2 pi = 6.28125, exact in
-    // few bits, plus a small remainder, so k * 6.28125 is exact), then the fast
-    // sine and cosine, whose documented error on that interval is 2^-21.4.
-    float ph = static_cast<float>(pos) * inv_freq;
-    const float k = rintf(ph * 0.15915494309189535f);
-    ph = fmaf(-k, 6.28125f, ph);
-    ph = fmaf(-k, 1.9353071795864769253e-3f, ph);
-    __sincosf(ph, &sn, &c);
+    turn_angle(pos, pair_inv_freq(i, da, p.log2_theta), c, sn);
     return true;
+}
+
+// One adjacent bf16 pair (x_a in the low half) turned by (c, sn).  Rounded
+// products and a fused add, spelled out so that every caller (this kernel and
+// the attention kernel's fused Q rotation) gets the same bits.
+__device__ __forceinline__ uint32_t rotate_pair(uint32_t word, float c, float sn)
+{
+    const __nv_bfloat162 e = *reinterpret_cast<const __nv_bfloat162 *>(&word);
+    const float xa = __low2float(e), xb = __high2float(e);
+    const __nv_bfloat162 o = __floats2bfloat162_rn(__fmaf_rn(xa, c, __fmul_rn(-xb, sn)),
+                                                   __fmaf_rn(xa, sn, __fmul_rn(xb, c)));
+    return *reinterpret_cast<const uint32_t *>(&o);
 }
 
 constexpr int ROPE_ROWS = 4;   // (b, h) rows loaded before any is stored
@@ -118,10 +152,7 @@ __device__ __forceinline__ void rope3d_vec_token(const RopeParams &p, int q4, in
             for (int k = 0; k < 4; ++k) {
                 if (!turn[k])
                     continue;   // copied bit for bit
-                const __nv_bfloat162 e = *reinterpret_cast<const __nv_bfloat162 *>(&w[k]);
-                const float xa = __low2float(e), xb = __high2float(e);
-                const __nv_bfloat162 o = __floats2bfloat162_rn(xa * c[k] - xb * sn[k], xa * sn[k] + xb * c[k]);
-                w[k] = *reinterpret_cast<const uint32_t *>(&o);
+                w[k] = rotate_pair(w[k], c[k], sn[k]);
             }
             *reinterpret_cast<uint4 *>(p.y + static_cast<size_t>(bh0 + r) * row_stride + off) =
                 make_uint4(w[0], w[1], w[2], w[3]);
@@ -179,8 +210,9 @@ __global__ void __launch_bounds__(256) rope3d_kernel(const RopeParams p)
             if (bh0 + r >= p.BH)
                 break;
             const size_t o = static_cast<size_t>(bh0 + r) * row_stride + off;
-            const float ya = turns ? xa[r] * c - xb[r] * sn : xa[r];   // bf16 -> fp32 -> bf16: exact copy
-            const float yb = turns ? xa[r] * sn + xb[r] * c : xb[r];
+            // bf16 -> fp32 -> bf16 is an exact copy; turned pairs as in rotate_pair
+            const float ya = turns ? __fmaf_rn(xa[r], c, __fmul_rn(-xb[r], sn)) : xa[r];
+            const float yb = turns ? __fmaf_rn(xa[r], sn, __fmul_rn(xb[r], c)) : xb[r];
             if (packed) {
                 *reinterpret_cast<__nv_bfloat162 *>(p.y + o + ia) = __floats2bfloat162_rn(ya, yb);
             } else {

@@ -17,6 +17,7 @@
 #include <cstring>
 #include <map>
 #include <mutex>
+#include <tuple>
 #include <utility>
 #include <vector>
 
@@ -138,13 +139,16 @@ struct Workspace {
     void *ptr = nullptr;
     size_t bytes = 0;
 };
+// kind: WS_TAIL (split tail, key-tile lists) or WS_ROPE_K / WS_ROPE_Q (the
+// turned K and Q of vdx_attn_fwd_rope3d).
+enum { WS_TAIL = 0, WS_ROPE_K = 1, WS_ROPE_Q = 2 };
 std::mutex g_ws_mutex;
-std::map<std::pair<int, cudaStream_t>, Workspace> g_ws;
+std::map<std::tuple<int, cudaStream_t, int>, Workspace> g_ws;
 
-int workspace(int dev, cudaStream_t stream, size_t bytes, void **out)
+int workspace(int dev, cudaStream_t stream, size_t bytes, void **out, int kind = WS_TAIL)
 {
     std::lock_guard<std::mutex> lock(g_ws_mutex);
-    Workspace &w = g_ws[{dev, stream}];
+    Workspace &w = g_ws[std::make_tuple(dev, stream, kind)];
     if (w.bytes < bytes) {
         if (w.ptr && cudaFree(w.ptr) != cudaSuccess)
             return VDX_ERR_CUDA;
@@ -368,14 +372,14 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     cudaError_t e;
     if (D == 128) {
         e = varlen ? launch<128, MODE_VARLEN, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
-                   : seg ? launch<128, MODE_SEG, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
-                         : win ? launch<128, MODE_WIN, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
-                               : launch<128, MODE_DENSE, 1, 2>(grid, mq, mk, mv, mo, p, sp, s);
+            : seg  ? launch<128, MODE_SEG, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
+            : win  ? launch<128, MODE_WIN, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
+                   : launch<128, MODE_DENSE, 1, 2>(grid, mq, mk, mv, mo, p, sp, s);
     } else {
         e = varlen ? launch<64, MODE_VARLEN, 2, 4>(grid, mq, mk, mv, mo, p, sp, s)
-                   : seg ? launch<64, MODE_SEG, 2, 4>(grid, mq, mk, mv, mo, p, sp, s)
-                         : win ? launch<64, MODE_WIN, 2, 4>(grid, mq, mk, mv, mo, p, sp, s)
-                               : launch<64, MODE_DENSE, 2, 4>(grid, mq, mk, mv, mo, p, sp, s);
+            : seg  ? launch<64, MODE_SEG, 2, 4>(grid, mq, mk, mv, mo, p, sp, s)
+            : win  ? launch<64, MODE_WIN, 2, 4>(grid, mq, mk, mv, mo, p, sp, s)
+                   : launch<64, MODE_DENSE, 2, 4>(grid, mq, mk, mv, mo, p, sp, s);
     }
     if (e == cudaErrorNoKernelImageForDevice)
         return VDX_ERR_DEVICE;
@@ -779,6 +783,76 @@ int host_pipeline(const void *q, const void *k, const void *v, void *out, float 
     return VDX_OK;
 }
 
+// Checks the arguments of a rotation (no CUDA calls) and fills p (p->BH == 0
+// or S == 0: nothing to do).
+int rope_args(const void *x, const void *y, int B, int H, int S, int D, int F, int Hp, int Wp, int s0, int d_t,
+              int d_h, int d_w, float theta, vdx::RopeParams *out_p)
+{
+    *out_p = vdx::RopeParams{};
+    if (!x || !y || B < 0 || H < 0 || S < 0 || F < 0 || Hp < 0 || Wp < 0 || s0 < 0)
+        return VDX_ERR_INVALID_ARG;
+    if (D < 2 || D > 512 || (D & 1) || d_t < 0 || d_h < 0 || d_w < 0 || ((d_t | d_h | d_w) & 1) ||
+        static_cast<long long>(d_t) + d_h + d_w > D)
+        return VDX_ERR_INVALID_ARG;
+    if (!std::isfinite(theta) || !(theta > 0.f))
+        return VDX_ERR_INVALID_ARG;
+    if (!aligned(x, 4) || !aligned(y, 4))
+        return VDX_ERR_MISALIGNED;
+    const long long bh = static_cast<long long>(B) * H;
+    if (bh > INT_MAX)
+        return VDX_ERR_INVALID_ARG;
+    const size_t bytes = static_cast<size_t>(bh) * S * D * 2;
+    if (x != y && overlaps(x, bytes, y, bytes))
+        return VDX_ERR_INVALID_ARG;
+    vdx::RopeParams p{};
+    p.x = static_cast<const __nv_bfloat16 *>(x);
+    p.y = static_cast<__nv_bfloat16 *>(const_cast<void *>(y));
+    p.BH = static_cast<int>(bh);
+    p.S = S;
+    p.D = D;
+    p.F = F;
+    p.Hp = Hp;
+    p.Wp = Wp;
+    p.s0 = s0;
+    p.d_t = d_t;
+    p.d_h = d_h;
+    p.d_w = d_w;
+    p.log2_theta = static_cast<float>(std::log2(static_cast<double>(theta)));
+    p.copy_all = x != y;
+    *out_p = p;
+    return VDX_OK;
+}
+
+// Launches the rotation p describes (validated by rope_args).
+int rope_launch(const vdx::RopeParams &p, bool interleaved, cudaStream_t s)
+{
+    int sms = 0;
+    const int st = device_ready(&sms);
+    if (st != VDX_OK)
+        return st;
+    const int D = p.D, S = p.S;
+    const void *x = p.x, *y = p.y;
+    if (interleaved && D % 8 == 0 && aligned(x, 16) && aligned(y, 16)) {
+        // 16-byte chunks: four pairs per thread
+        const int chunks = D / 8;
+        const int tok = 256 / chunks;
+        const long long groups = (S + tok - 1) / tok;
+        const long long cap = static_cast<long long>(sms) * vdx::ROPE_VEC_BLOCKS_PER_SM;
+        const unsigned nb = static_cast<unsigned>(groups < cap ? groups : cap);
+        vdx::rope3d_vec_kernel<<<dim3(nb), dim3(static_cast<unsigned>(chunks), static_cast<unsigned>(tok)), 0, s>>>(p);
+    } else {
+        const int pairs = D / 2;
+        const int tok = 256 / pairs;
+        const dim3 block(static_cast<unsigned>(pairs), static_cast<unsigned>(tok));
+        const dim3 grid(static_cast<unsigned>((S + tok - 1) / tok));
+        if (interleaved)
+            vdx::rope3d_kernel<true><<<grid, block, 0, s>>>(p);
+        else
+            vdx::rope3d_kernel<false><<<grid, block, 0, s>>>(p);
+    }
+    return cudaGetLastError() == cudaSuccess ? VDX_OK : VDX_ERR_CUDA;
+}
+
 }  // namespace
 
 extern "C" {
@@ -866,64 +940,53 @@ int vdx_attn_fwd_win3d(const void *q, const void *k, const void *v, void *out, f
 int vdx_rope3d(const void *x, void *y, int B, int H, int S, int D, int F, int Hp, int Wp, int s0, int d_t, int d_h,
                int d_w, float theta, int interleaved, void *stream)
 {
-    // ---- validation (no CUDA calls)
-    if (!x || !y || B < 0 || H < 0 || S < 0 || F < 0 || Hp < 0 || Wp < 0 || s0 < 0)
-        return VDX_ERR_INVALID_ARG;
-    if (D < 2 || D > 512 || (D & 1) || d_t < 0 || d_h < 0 || d_w < 0 || ((d_t | d_h | d_w) & 1) ||
-        static_cast<long long>(d_t) + d_h + d_w > D)
-        return VDX_ERR_INVALID_ARG;
-    if (!std::isfinite(theta) || !(theta > 0.f))
-        return VDX_ERR_INVALID_ARG;
-    if (!aligned(x, 4) || !aligned(y, 4))
-        return VDX_ERR_MISALIGNED;
-    const long long bh = static_cast<long long>(B) * H;
-    if (bh == 0 || S == 0)
-        return VDX_OK;
-    if (bh > INT_MAX)
-        return VDX_ERR_INVALID_ARG;
-    const size_t bytes = static_cast<size_t>(bh) * S * D * 2;
-    if (x != y && overlaps(x, bytes, y, bytes))
-        return VDX_ERR_INVALID_ARG;
-    // ---- device set-up and launch
-    int sms = 0;
-    const int st = device_ready(&sms);
+    vdx::RopeParams p{};
+    const int st = rope_args(x, y, B, H, S, D, F, Hp, Wp, s0, d_t, d_h, d_w, theta, &p);
+    if (st != VDX_OK || p.BH == 0 || S == 0)
+        return st;
+    return rope_launch(p, interleaved != 0, static_cast<cudaStream_t>(stream));
+}
+
+int vdx_attn_fwd_rope3d(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int S,
+                        int D, int F, int Hp, int Wp, int s0, int d_t, int d_h, int d_w, float theta,
+                        int interleaved, float scale, void *stream)
+{
+    // ---- validation: the rotation's and the attention's (no CUDA calls)
+    vdx::RopeParams rq{}, rk{};
+    int st = rope_args(q, q, B, H, S, D, F, Hp, Wp, s0, d_t, d_h, d_w, theta, &rq);
     if (st != VDX_OK)
         return st;
-    vdx::RopeParams p{};
-    p.x = static_cast<const __nv_bfloat16 *>(x);
-    p.y = static_cast<__nv_bfloat16 *>(y);
-    p.BH = static_cast<int>(bh);
-    p.S = S;
-    p.D = D;
-    p.F = F;
-    p.Hp = Hp;
-    p.Wp = Wp;
-    p.s0 = s0;
-    p.d_t = d_t;
-    p.d_h = d_h;
-    p.d_w = d_w;
-    p.log2_theta = static_cast<float>(std::log2(static_cast<double>(theta)));
-    p.copy_all = x != y;
+    if ((st = rope_args(k, k, B, H, S, D, F, Hp, Wp, s0, d_t, d_h, d_w, theta, &rk)) != VDX_OK)
+        return st;
+    if (!v || !out || !std::isfinite(scale) || (D != 64 && D != 128))
+        return VDX_ERR_INVALID_ARG;
+    if (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(out, 16) || (lse && !aligned(lse, 4)))
+        return VDX_ERR_MISALIGNED;
+    const size_t bytes = static_cast<size_t>(rk.BH) * S * D * 2;
+    if (rk.BH == 0 || S == 0)
+        return VDX_OK;
+    if (overlaps(out, bytes, q, bytes) || overlaps(out, bytes, k, bytes) || overlaps(out, bytes, v, bytes))
+        return VDX_ERR_INVALID_ARG;
+
+    // ---- Q and K turned by the RoPE kernel into the library's per-stream
+    // buffers, then the dense attention on them
+    int sms = 0, dev = 0;
+    if ((st = device_ready(&sms)) != VDX_OK)
+        return st;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return VDX_ERR_CUDA;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    if (interleaved && D % 8 == 0 && aligned(x, 16) && aligned(y, 16)) {
-        // 16-byte chunks: four pairs per thread
-        const int chunks = D / 8;
-        const int tok = 256 / chunks;
-        const long long groups = (S + tok - 1) / tok;
-        const long long cap = static_cast<long long>(sms) * vdx::ROPE_VEC_BLOCKS_PER_SM;
-        const unsigned nb = static_cast<unsigned>(groups < cap ? groups : cap);
-        vdx::rope3d_vec_kernel<<<dim3(nb), dim3(static_cast<unsigned>(chunks), static_cast<unsigned>(tok)), 0, s>>>(p);
-    } else {
-        const int pairs = D / 2;
-        const int tok = 256 / pairs;
-        const dim3 block(static_cast<unsigned>(pairs), static_cast<unsigned>(tok));
-        const dim3 grid(static_cast<unsigned>((S + tok - 1) / tok));
-        if (interleaved)
-            vdx::rope3d_kernel<true><<<grid, block, 0, s>>>(p);
-        else
-            vdx::rope3d_kernel<false><<<grid, block, 0, s>>>(p);
-    }
-    return cudaGetLastError() == cudaSuccess ? VDX_OK : VDX_ERR_CUDA;
+    void *q_rot = nullptr, *k_rot = nullptr;
+    if ((st = workspace(dev, s, bytes, &q_rot, WS_ROPE_Q)) != VDX_OK ||
+        (st = workspace(dev, s, bytes, &k_rot, WS_ROPE_K)) != VDX_OK)
+        return st;
+    rq.y = static_cast<__nv_bfloat16 *>(q_rot);
+    rq.copy_all = 1;
+    rk.y = static_cast<__nv_bfloat16 *>(k_rot);
+    rk.copy_all = 1;
+    if ((st = rope_launch(rq, interleaved != 0, s)) != VDX_OK || (st = rope_launch(rk, interleaved != 0, s)) != VDX_OK)
+        return st;
+    return attn_launch(q_rot, k_rot, v, out, lse, B, H, S, S, D, KeyRule{}, scale, stream);
 }
 
 int vdx_attn_fwd_segments(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,

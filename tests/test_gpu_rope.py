@@ -88,3 +88,62 @@ def test_rope_not_16_byte_aligned():
     y = binding.rope3d(xs, grid, s0, (44, 42, 42), 1e4, True)
     assert binding.check_device_error() == binding.VDX_OK
     _check(y, x, y_ref)
+
+
+# RoPE + attention in one call: B, H, D, grid, s0, tokens after the grid, dims, theta, interleaved
+ROPE_ATTN = [
+    (1, 3, 128, (3, 5, 7), 0, 0, (44, 42, 42), 1e4, True),       # S = 105: one ragged query tile pair
+    (2, 2, 128, (4, 6, 11), 20, 13, (44, 42, 42), 1e4, True),    # text before, tokens after the grid
+    (1, 2, 64, (5, 8, 9), 7, 0, (24, 20, 20), 1e4, True),         # D = 64 (two Q buffers)
+    (1, 2, 128, (2, 9, 20), 0, 5, (16, 16, 16), 300.0, True),     # dims past the rotated parts unturned
+    (1, 2, 128, (3, 5, 7), 3, 2, (44, 42, 42), 1e4, False),      # half-split pairs
+    (1, 1, 128, (8, 16, 16), 0, 0, (44, 42, 42), 1e4, True),      # 2048 tokens: several units per CTA
+]
+
+
+@pytest.mark.parametrize("B,H,D,grid,s0,after,dims,theta,inter", ROPE_ATTN)
+def test_rope_attention_bit_identical_to_separate_calls(B, H, D, grid, s0, after, dims, theta, inter):
+    """vdx_attn_fwd_rope3d gives, bit for bit, vdx_rope3d on q and k followed
+    by vdx_attn_fwd, leaves q and k untouched, and matches the oracle."""
+    import oracle
+    S = s0 + grid[0] * grid[1] * grid[2] + after
+    q, k, v = workloads.random_qkv(B, H, S, S, D, seed=800 + S + D, logit_gain=1.5)
+    qd, kd, vd = q.cuda(), k.cuda(), v.cuda()
+    scale = D ** -0.5
+    out, lse = binding.attn_fwd_rope3d(qd, kd, vd, grid, s0, dims, theta, inter, scale=scale)
+    assert binding.check_device_error() == binding.VDX_OK
+    assert torch.equal(qd.cpu().view(torch.int16), q.view(torch.int16))
+    assert torch.equal(kd.cpu().view(torch.int16), k.view(torch.int16))
+    qr = binding.rope3d(qd, grid, s0, dims, theta, inter)
+    kr = binding.rope3d(kd, grid, s0, dims, theta, inter)
+    o_sep, l_sep = binding.attn_fwd(qr, kr, vd, scale=scale)
+    assert torch.equal(out, o_sep)
+    assert torch.equal(lse, l_sep)
+    from parity import compare
+    q_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(q), grid, s0, dims, theta, inter)).to(torch.bfloat16)
+    k_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(k), grid, s0, dims, theta, inter)).to(torch.bfloat16)
+    o_ref, lse_ref = oracle.attn_fwd(workloads.bf16_bits(q_ref), workloads.bf16_bits(k_ref), workloads.bf16_bits(v),
+                                     scale)
+    compare(out, lse, o_ref, lse_ref)
+
+
+def test_rope_attention_rope480():
+    """The rope480 workload through the one call: bit for bit the separate
+    calls, and the oracle on a seeded row sample."""
+    import oracle
+    from parity import compare
+    w = workloads.generate("rope480")
+    grid, s0, dims, theta, inter = w["workload"].rope
+    qd, kd, vd = (w[n].cuda() for n in ("q", "k", "v"))
+    out, lse = binding.attn_fwd_rope3d(qd, kd, vd, grid, s0, dims, theta, inter, scale=w["scale"])
+    o_sep, l_sep = binding.attn_fwd(binding.rope3d(qd, grid, s0, dims, theta, inter),
+                                    binding.rope3d(kd, grid, s0, dims, theta, inter), vd, scale=w["scale"])
+    assert torch.equal(out, o_sep) and torch.equal(lse, l_sep)
+    rows = np.ascontiguousarray(w["rows"][:, :256])
+    q_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(w["q"]), grid, s0, dims, theta, inter)).to(torch.bfloat16)
+    k_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(w["k"]), grid, s0, dims, theta, inter)).to(torch.bfloat16)
+    o_ref, lse_ref = oracle.attn_fwd(workloads.bf16_bits(q_ref), workloads.bf16_bits(k_ref), workloads.bf16_bits(w["v"]),
+                                     w["scale"], rows=rows)
+    compare(out, lse, o_ref, lse_ref, rows)
+    del out, lse, o_sep, l_sep
+    torch.cuda.empty_cache()

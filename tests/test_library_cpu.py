@@ -174,3 +174,24 @@ def test_segment_and_window_host_entries_validate(lib):
     from paper_2609_18077_gb300 import binding
     with pytest.raises(TypeError):
         binding.attn_fwd_segments_host(q, q, q, ids, torch.zeros(1, 7, dtype=torch.int32))
+
+
+def test_rope_attention_validates(lib):
+    """vdx_attn_fwd_rope3d rejects bad arguments before any CUDA call."""
+    g = GOOD
+    f = lib.vdx_attn_fwd_rope3d
+    base = dict(B=1, H=1, S=8, D=128, F=2, Hp=2, Wp=2, s0=0, dt=44, dh=42, dw=42, theta=1e4, inter=1, scale=0.1)
+
+    def call(**kw):
+        a = {**base, **kw}
+        return f(g["q"], g["k"], g["v"], g["out"], g["lse"], a["B"], a["H"], a["S"], a["D"], a["F"], a["Hp"],
+                 a["Wp"], a["s0"], a["dt"], a["dh"], a["dw"], a["theta"], a["inter"], a["scale"], None)
+    assert call(D=96, dt=32, dh=32, dw=32) == 1       # attention needs D 64 or 128
+    assert call(dt=45) == 1                            # odd part
+    assert call(dt=64, dh=64, dw=8) == 1               # parts wider than D
+    assert call(theta=-1.0) == 1
+    assert call(scale=float("nan")) == 1
+    assert call(B=-1) == 1
+    assert call(S=0) == 0                              # nothing to do
+    assert f(g["q"] + 8, g["k"], g["v"], g["out"], g["lse"], 1, 1, 8, 128, 2, 2, 2, 0, 44, 42, 42, 1e4, 1, 0.1,
+             None) == 3                                # q not 16-byte aligned
