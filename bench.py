@@ -197,8 +197,7 @@ def run_ours(args):
 
     # ---- device-resident timed region
     peaks, peak_kind = load_peaks()
-    clocks_log = os.path.join(ROOT, "gpurun_out", "bench_clocks.csv") if os.path.isdir(
-        os.path.join(ROOT, "gpurun_out")) else None
+    clocks_log = os.environ.get("VDX_BENCH_CLOCKS_CSV") or None   # optional raw nvidia-smi samples
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local, clocks_log) as clk:
         barrier()
