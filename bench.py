@@ -335,14 +335,20 @@ def run_ours(args):
 
 
 def kernel_source_hash():
-    """sha256 over the CUDA sources, to tell whether a stored ncu capture still applies."""
+    """sha256 over the CUDA sources' code (comments and whitespace removed), to
+    tell whether a stored ncu capture still applies to the kernels."""
     import hashlib
+    import re
     csrc = os.path.join(ROOT, "paper_2609_18077_gb300", "csrc")
     h = hashlib.sha256()
     for name in sorted(os.listdir(csrc)):
         if name.endswith((".cu", ".cuh", ".h")):
-            with open(os.path.join(csrc, name), "rb") as f:
-                h.update(name.encode() + b"\0" + f.read())
+            with open(os.path.join(csrc, name)) as f:
+                code = f.read()
+            code = re.sub(r"/\*.*?\*/", " ", code, flags=re.S)   # block comments
+            code = re.sub(r"//[^\n]*", " ", code)                  # line comments
+            code = "".join(code.split())                            # whitespace
+            h.update(name.encode() + b"\0" + code.encode())
     return h.hexdigest()[:16]
 
 

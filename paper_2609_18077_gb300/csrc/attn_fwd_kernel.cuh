@@ -10,7 +10,10 @@
 // segment instance (joint text-video attention, same appendix entry) lets
 // query i attend key j iff their segment ids match: each unit visits only the
 // key tiles of its list (segment_tiles.cuh) and compares ids element by
-// element only on the tiles the list marks.
+// element only on the tiles the list marks.  The window instance (windowed 3D
+// attention, appendix Table 4's VAE decoder) walks per query-tile-pair lists
+// of the key tiles inside the unit's window box (window_tiles.cuh) and masks
+// keys outside each row's window.
 //
 // Work unit: one (b*h, pair of 128-row query tiles).  The grid is persistent:
 // one CTA per SM walks the units u = blockIdx.x, blockIdx.x + gridDim.x, ...
@@ -23,7 +26,8 @@
 //   warps 4-7  softmax of query tile 1
 //   warp  8    TMA producer: Q tiles once, then K_0 and the stages
 //              (V_0, K_1), (V_1, K_2), ... through a ring of NSTAGE
-//              two-tile stages (one full and one empty barrier per stage)
+//              two-tile stages (one full and one empty barrier per stage);
+//              the next unit's Q tiles are prefetched into L2 meanwhile
 //   warp  9    tcgen05 issuer (one lane) and TMEM owner
 // Tensor memory (512 columns x 128 lanes, fp32):
 //   S_t = cols [128t, 128t+128): logits Q_t K_j^T; the probabilities P_t are
@@ -48,6 +52,11 @@
 // that tile's largest weight in the row.  That makes the dominant weight
 // exact at the cost of a few instructions per tile; the log-sum-exp uses the
 // exact sum alone.
+//
+// Epilogue: O / l packed to bf16 by the softmax threads, one row each, and
+// stored per thread; the text cross-attention instance, whose units are a few
+// key tiles long, stores it through per-warp TMA stores from swizzled staging
+// boxes instead (stages_out below).
 //
 // Every wait is bounded (globaltimer); on expiry the CTA records
 // VDX_ERR_TIMEOUT in the device error word, skips the rest of its work, frees
