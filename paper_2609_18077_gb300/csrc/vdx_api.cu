@@ -713,22 +713,31 @@ int host_pipeline(const void *q, const void *k, const void *v, void *out, float 
         return base + lens_b + static_cast<size_t>(i) * slot_b + off[part];
     };
 
-    // ---- enqueue: everything after the caller's earlier work on `stream`
+    // ---- enqueue: everything after the caller's earlier work on `stream`.
+    // A failure after the first enqueue still makes `stream` wait for all the
+    // pipeline's streams, so that no later call reuses a slot under work in
+    // flight.
+    auto fail = [&](int code) {
+        for (cudaStream_t own : {pp.up, pp.run[0], pp.run[1], pp.down})
+            if (cudaEventRecord(pp.start, own) == cudaSuccess)
+                (void)cudaStreamWaitEvent(s, pp.start, 0);
+        return code;
+    };
     const char *qh = static_cast<const char *>(q), *kh = static_cast<const char *>(k);
     const char *vh = static_cast<const char *>(v);
     char *oh = static_cast<char *>(out), *lh = reinterpret_cast<char *>(lse);
     if (cudaEventRecord(pp.start, s) != cudaSuccess || cudaStreamWaitEvent(pp.up, pp.start, 0) != cudaSuccess ||
         cudaStreamWaitEvent(pp.run[0], pp.start, 0) != cudaSuccess ||
         cudaStreamWaitEvent(pp.run[1], pp.start, 0) != cudaSuccess)
-        return VDX_ERR_CUDA;
+        return fail(VDX_ERR_CUDA);
     if (varlen && cudaMemcpyAsync(d_lens, hr.kv_lens, static_cast<size_t>(B) * 4, cudaMemcpyHostToDevice, pp.up) !=
                       cudaSuccess)
-        return VDX_ERR_CUDA;
+        return fail(VDX_ERR_CUDA);
     if (seg && (cudaMemcpyAsync(d_qseg, hr.q_seg, static_cast<size_t>(B) * Sq * 4, cudaMemcpyHostToDevice, pp.up) !=
                     cudaSuccess ||
                 (Skv > 0 && cudaMemcpyAsync(d_kvseg, hr.kv_seg, static_cast<size_t>(B) * Skv * 4,
                                             cudaMemcpyHostToDevice, pp.up) != cudaSuccess)))
-        return VDX_ERR_CUDA;
+        return fail(VDX_ERR_CUDA);
     const size_t n = chunks.size();
     for (size_t i = 0; i <= n; ++i) {
         if (i < n) {
@@ -738,7 +747,7 @@ int host_pipeline(const void *q, const void *k, const void *v, void *out, float 
             const int sl = static_cast<int>(i % kHostSlots);
             cudaStream_t rs = pp.run[i & 1];
             if (i >= kHostSlots && cudaStreamWaitEvent(pp.up, pp.comp[sl], 0) != cudaSuccess)
-                return VDX_ERR_CUDA;
+                return fail(VDX_ERR_CUDA);
             const size_t nq = c.rows * row_q, nkv = c.rows * row_kv;
             if (cudaMemcpyAsync(slot(sl, 0), qh + c.row0 * row_q, nq, cudaMemcpyHostToDevice, pp.up) != cudaSuccess ||
                 (nkv && (cudaMemcpyAsync(slot(sl, 1), kh + c.row0 * row_kv, nkv, cudaMemcpyHostToDevice, pp.up) !=
@@ -748,7 +757,7 @@ int host_pipeline(const void *q, const void *k, const void *v, void *out, float 
                 cudaEventRecord(pp.h2d[sl], pp.up) != cudaSuccess ||
                 cudaStreamWaitEvent(rs, pp.h2d[sl], 0) != cudaSuccess ||
                 (i >= kHostSlots && cudaStreamWaitEvent(rs, pp.d2h[sl], 0) != cudaSuccess))
-                return VDX_ERR_CUDA;
+                return fail(VDX_ERR_CUDA);
             KeyRule rule = hr;   // window problems: the grid as given
             if (varlen)
                 rule.kv_lens = d_lens + c.b0;
@@ -760,9 +769,9 @@ int host_pipeline(const void *q, const void *k, const void *v, void *out, float 
                              lse ? reinterpret_cast<float *>(slot(sl, 4)) : nullptr, c.nb, c.nh, Sq, Skv, D, rule,
                              scale, rs);
             if (st != VDX_OK)
-                return st;
+                return fail(st);
             if (cudaEventRecord(pp.comp[sl], rs) != cudaSuccess)
-                return VDX_ERR_CUDA;
+                return fail(VDX_ERR_CUDA);
         }
         if (i >= 1) {
             // copy chunk i-1 out once its kernel is done
@@ -774,12 +783,12 @@ int host_pipeline(const void *q, const void *k, const void *v, void *out, float 
                 (lse && cudaMemcpyAsync(lh + c.row0 * row_l, slot(sl, 4), c.rows * row_l, cudaMemcpyDeviceToHost,
                                         pp.down) != cudaSuccess) ||
                 cudaEventRecord(pp.d2h[sl], pp.down) != cudaSuccess)
-                return VDX_ERR_CUDA;
+                return fail(VDX_ERR_CUDA);
         }
     }
     // the caller's stream resumes once the last result is on the host
     if (cudaStreamWaitEvent(s, pp.d2h[(n - 1) % kHostSlots], 0) != cudaSuccess)
-        return VDX_ERR_CUDA;
+        return fail(VDX_ERR_CUDA);
     return VDX_OK;
 }
 
