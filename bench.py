@@ -18,9 +18,8 @@ L2, so no flush is inserted.  SM clocks are sampled with nvidia-smi during
 the timed region.  A second timed pass ("e2e") starts from pinned host
 buffers: every step copies Q, K, V host->device, runs the kernel and copies
 O and LSE back.  Each step is one host-buffer call (vdx_attn_fwd_host, or its
-segment or window variant: the library cuts the (b, h) rows into chunks and
-overlaps the copies with the kernel); the RoPE workload copies, runs its
-three kernels and copies back in turn.
+segment, window or RoPE variant): the library cuts the (b, h) rows into
+chunks and overlaps the copies with the kernels.
 
 --impl reference times the fp64 CPU oracle (the only reference this
 method has) on a bounded row sample of the same workload.  Under torchrun
@@ -248,32 +247,21 @@ def run_ours(args):
         (0 if sh is None else sum(t.numel() * 4 for t in sh))
     d2h = oh.numel() * oh.element_size() + lseh.numel() * lseh.element_size()
 
-    host_api = wl.rope is None
-
     def e2e_step():
-        if host_api:
-            # one host-buffer call: chunked, copies overlapped with the kernel
-            if wl.window is not None:
-                binding.attn_fwd_win3d_host(qh, kh, vh, wl.latent, wl.window[0], wl.window[1], scale=wl.scale,
-                                            out=oh, lse=lseh, device=dev, synchronize=False)
-            elif sh is not None:
-                binding.attn_fwd_segments_host(qh, kh, vh, sh[0], sh[1], scale=wl.scale, out=oh, lse=lseh,
-                                               device=dev, synchronize=False)
-            else:
-                binding.attn_fwd_host(qh, kh, vh, kv_lens=lh, scale=wl.scale, out=oh, lse=lseh, device=dev,
-                                      synchronize=False)
-            return
-        q.copy_(qh, non_blocking=True)
-        k.copy_(kh, non_blocking=True)
-        v.copy_(vh, non_blocking=True)
-        if lh is not None:
-            lens.copy_(lh, non_blocking=True)
-        if sh is not None:
-            segs[0].copy_(sh[0], non_blocking=True)
-            segs[1].copy_(sh[1], non_blocking=True)
-        step()
-        oh.copy_(out, non_blocking=True)
-        lseh.copy_(lse, non_blocking=True)
+        # one host-buffer call: chunks of (b, h) rows, copies overlapped with the kernels
+        if rope is not None:
+            grid, s0, dims, theta, inter = rope
+            binding.attn_fwd_rope3d_host(qh, kh, vh, grid, s0, dims, theta, inter, scale=wl.scale, out=oh,
+                                         lse=lseh, device=dev, synchronize=False)
+        elif wl.window is not None:
+            binding.attn_fwd_win3d_host(qh, kh, vh, wl.latent, wl.window[0], wl.window[1], scale=wl.scale,
+                                        out=oh, lse=lseh, device=dev, synchronize=False)
+        elif sh is not None:
+            binding.attn_fwd_segments_host(qh, kh, vh, sh[0], sh[1], scale=wl.scale, out=oh, lse=lseh,
+                                           device=dev, synchronize=False)
+        else:
+            binding.attn_fwd_host(qh, kh, vh, kv_lens=lh, scale=wl.scale, out=oh, lse=lseh, device=dev,
+                                  synchronize=False)
 
     e2e_steps = max(3, min(args.steps, 50))
     for _ in range(2):
@@ -315,11 +303,10 @@ def run_ours(args):
         "clocks": clocks,
         "e2e": {"value": round(e2e_tflops, 2), "unit": UNIT, "ms_per_step": round(e2e_ms, 4),
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
-                "path": ("host-buffer entry point (vdx_attn_fwd%s_host): pinned host buffers, chunks of (b, h) "
-                         "rows, copies in and out overlapped with the kernel" % (
-                             "_win3d" if wl.window is not None else ("_segments" if sh is not None else ""))
-                         if host_api else
-                         "pinned host buffers copied in, the step's kernels, results copied out")},
+                "path": "host-buffer entry point (vdx_attn_fwd%s_host): pinned host buffers, chunks of (b, h) "
+                        "rows, copies in and out overlapped with the kernels" % (
+                            "_rope3d" if rope is not None else
+                            ("_win3d" if wl.window is not None else ("_segments" if sh is not None else "")))},
         "gpu_launches": args.steps * launches_per_step,
         "roofline": {"bound": "tensor", "achieved": round(per_launch_tflops, 2), "peak": peak,
                      "unit": "TFLOP/s", "frac": round(per_launch_tflops / peak, 4),

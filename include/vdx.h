@@ -232,6 +232,20 @@ int vdx_attn_fwd_host(const void *q, const void *k, const void *v, void *out, fl
                       long long chunk_rows, void *stream);
 
 /*
+ * vdx_attn_fwd_rope3d on HOST buffers, through the same pipeline as
+ * vdx_attn_fwd_host: each chunk's q and k rows are turned in place in the
+ * device slot (the rotation works row by row, so a chunk turns exactly as
+ * the whole tensor would) before the chunk's attention.  Arguments as
+ * vdx_attn_fwd_rope3d plus chunk_rows; results: each chunk is vdx_rope3d on
+ * its q and k rows followed by vdx_attn_fwd on those rows.  Errors as
+ * vdx_attn_fwd_rope3d and vdx_attn_fwd_host.
+ */
+int vdx_attn_fwd_rope3d_host(const void *q, const void *k, const void *v, void *out, float *lse,
+                             int B, int H, int S, int D, int F, int Hp, int Wp, int s0,
+                             int d_t, int d_h, int d_w, float theta, int interleaved,
+                             float scale, long long chunk_rows, void *stream);
+
+/*
  * vdx_attn_fwd_segments on HOST buffers, through the same pipeline as
  * vdx_attn_fwd_host.  q_seg [B, Sq] and kv_seg [B, Skv] are HOST int32
  * arrays, copied in once per call; chunks hold heads of one sample or whole

@@ -40,6 +40,8 @@ SIGNATURES = {
     "vdx_attn_fwd_segments_host": (_I, [_P, _P, _P, _P, _P, _I, _I, _I, _I, _I, _P, _P, ctypes.c_float,
                                         ctypes.c_longlong, _P]),
     "vdx_attn_fwd_win3d_host": (_I, [_P, _P, _P, _P, _P] + [_I] * 10 + [ctypes.c_float, ctypes.c_longlong, _P]),
+    "vdx_attn_fwd_rope3d_host": (_I, [_P, _P, _P, _P, _P] + [_I] * 11 + [ctypes.c_float, _I, ctypes.c_float,
+                                                                         ctypes.c_longlong, _P]),
     "vdx_status_string": (ctypes.c_char_p, [_I]),
     "vdx_check_device_error": (_I, [_P]),
     "vdx_selftest_wait_timeout": (_I, [_I, _P]),
@@ -368,4 +370,24 @@ def attn_fwd_win3d_host(q, k, v, grid, window, neighbourhood=True, scale=None, o
                (q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
                 lse.data_ptr() if lse is not None else None, B, H, F, Hp, Wp, D, int(window[0]), int(window[1]),
                 int(window[2]), int(bool(neighbourhood)), scale, int(chunk_rows)), device, synchronize)
+    return out, lse
+
+
+def attn_fwd_rope3d_host(q, k, v, grid, s0, dims, theta, interleaved=True, scale=None, out=None, lse=None,
+                         return_lse=True, chunk_rows=0, device=None, synchronize=True):
+    """attn_fwd_rope3d on host tensors through ``vdx_attn_fwd_rope3d_host``
+    (each chunk's q and k rows turned in the device slot, then attended).
+    Other arguments as attn_fwd_host."""
+    _host_check(q, k, v)
+    B, H, S, D = q.shape
+    if k.shape[2] != S:
+        raise ValueError("q and k must hold the same tokens")
+    F, Hp, Wp = (int(x) for x in grid)
+    d_t, d_h, d_w = (int(x) for x in dims)
+    out, lse = _host_outputs(q, out, lse, return_lse)
+    scale = 1.0 / math.sqrt(D) if scale is None else float(scale)
+    _host_call(load().vdx_attn_fwd_rope3d_host, "vdx_attn_fwd_rope3d_host",
+               (q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(),
+                lse.data_ptr() if lse is not None else None, B, H, S, D, F, Hp, Wp, int(s0), d_t, d_h, d_w,
+                float(theta), int(bool(interleaved)), scale, int(chunk_rows)), device, synchronize)
     return out, lse

@@ -445,6 +445,8 @@ int win_rule(int F, int Hp, int Wp, int kt, int kh, int kw, int neighbourhood, K
     return VDX_OK;
 }
 
+int rope_launch(const vdx::RopeParams &p, bool interleaved, cudaStream_t s);   // the 3D RoPE, below
+
 // ---------------------------------------------------------------- host-buffer pipeline
 // vdx_attn_fwd_host cuts the (b, h) rows into chunks.  Chunk i is copied in
 // on one stream, run on one of two compute streams (alternating, so that
@@ -643,7 +645,8 @@ long long auto_chunk_rows(int B, int H, int Sq, int Skv, int D, const int *kv_le
 // [B]; q_seg [B, Sq] and kv_seg [B, Skv]); they are copied to the device once
 // per call.  Window problems share one grid, so their chunks are any rows.
 int host_pipeline(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
-                  int D, const KeyRule &hr, float scale, long long chunk_rows, void *stream)
+                  int D, const KeyRule &hr, float scale, long long chunk_rows, void *stream,
+                  const vdx::RopeParams *rope = nullptr, bool rope_interleaved = true)
 {
     // ---- validation (no CUDA calls)
     const bool varlen = hr.mode == vdx::MODE_VARLEN, seg = hr.mode == vdx::MODE_SEG;
@@ -758,6 +761,21 @@ int host_pipeline(const void *q, const void *k, const void *v, void *out, float 
                 cudaStreamWaitEvent(rs, pp.h2d[sl], 0) != cudaSuccess ||
                 (i >= kHostSlots && cudaStreamWaitEvent(rs, pp.d2h[sl], 0) != cudaSuccess))
                 return fail(VDX_ERR_CUDA);
+            if (rope) {
+                // the 3D RoPE of the chunk's q and k, in place in the slot (row by row,
+                // so a chunk of rows turns exactly as the whole tensor would)
+                vdx::RopeParams rq = *rope;
+                rq.BH = c.rows;
+                rq.copy_all = 0;
+                rq.S = Sq;
+                rq.x = rq.y = reinterpret_cast<__nv_bfloat16 *>(slot(sl, 0));
+                vdx::RopeParams rk = rq;
+                rk.S = Skv;
+                rk.x = rk.y = reinterpret_cast<__nv_bfloat16 *>(slot(sl, 1));
+                if ((st = rope_launch(rq, rope_interleaved, rs)) != VDX_OK ||
+                    (st = rope_launch(rk, rope_interleaved, rs)) != VDX_OK)
+                    return fail(st);
+            }
             KeyRule rule = hr;   // window problems: the grid as given
             if (varlen)
                 rule.kv_lens = d_lens + c.b0;
@@ -792,18 +810,21 @@ int host_pipeline(const void *q, const void *k, const void *v, void *out, float 
     return VDX_OK;
 }
 
+// The rotation's grid, head-dim split and base, pointers aside.
+bool rope_dims_ok(int D, int F, int Hp, int Wp, int s0, int d_t, int d_h, int d_w, float theta)
+{
+    return F >= 0 && Hp >= 0 && Wp >= 0 && s0 >= 0 && D >= 2 && D <= 512 && !(D & 1) && d_t >= 0 && d_h >= 0 &&
+           d_w >= 0 && !((d_t | d_h | d_w) & 1) && static_cast<long long>(d_t) + d_h + d_w <= D &&
+           std::isfinite(theta) && theta > 0.f;
+}
+
 // Checks the arguments of a rotation (no CUDA calls) and fills p (p->BH == 0
 // or S == 0: nothing to do).
 int rope_args(const void *x, const void *y, int B, int H, int S, int D, int F, int Hp, int Wp, int s0, int d_t,
               int d_h, int d_w, float theta, vdx::RopeParams *out_p)
 {
     *out_p = vdx::RopeParams{};
-    if (!x || !y || B < 0 || H < 0 || S < 0 || F < 0 || Hp < 0 || Wp < 0 || s0 < 0)
-        return VDX_ERR_INVALID_ARG;
-    if (D < 2 || D > 512 || (D & 1) || d_t < 0 || d_h < 0 || d_w < 0 || ((d_t | d_h | d_w) & 1) ||
-        static_cast<long long>(d_t) + d_h + d_w > D)
-        return VDX_ERR_INVALID_ARG;
-    if (!std::isfinite(theta) || !(theta > 0.f))
+    if (!x || !y || B < 0 || H < 0 || S < 0 || !rope_dims_ok(D, F, Hp, Wp, s0, d_t, d_h, d_w, theta))
         return VDX_ERR_INVALID_ARG;
     if (!aligned(x, 4) || !aligned(y, 4))
         return VDX_ERR_MISALIGNED;
@@ -909,6 +930,26 @@ int vdx_attn_fwd_host(const void *q, const void *k, const void *v, void *out, fl
         rule.kv_lens = kv_lens;
     }
     return host_pipeline(q, k, v, out, lse, B, H, Sq, Skv, D, rule, scale, chunk_rows, stream);
+}
+
+int vdx_attn_fwd_rope3d_host(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int S,
+                             int D, int F, int Hp, int Wp, int s0, int d_t, int d_h, int d_w, float theta,
+                             int interleaved, float scale, long long chunk_rows, void *stream)
+{
+    if (!rope_dims_ok(D, F, Hp, Wp, s0, d_t, d_h, d_w, theta))
+        return VDX_ERR_INVALID_ARG;
+    vdx::RopeParams rp{};
+    rp.D = D;
+    rp.F = F;
+    rp.Hp = Hp;
+    rp.Wp = Wp;
+    rp.s0 = s0;
+    rp.d_t = d_t;
+    rp.d_h = d_h;
+    rp.d_w = d_w;
+    rp.log2_theta = static_cast<float>(std::log2(static_cast<double>(theta)));
+    return host_pipeline(q, k, v, out, lse, B, H, S, S, D, KeyRule{}, scale, chunk_rows, stream, &rp,
+                         interleaved != 0);
 }
 
 int vdx_attn_fwd_segments_host(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H,

@@ -161,3 +161,32 @@ def test_win3d_host_bit_identical_to_one_device_call(r):
     assert torch.equal(lse, l_dev.cpu())
     o_ref, lse_ref = run_oracle(q, k, v, scale, window=(grid, window, True))
     compare(out, lse, o_ref, lse_ref)
+
+
+@pytest.mark.parametrize("r", [0, 1, 3, 6])
+def test_rope3d_host_bit_identical_to_device_chunks(r):
+    """Each chunk turns its q and k rows in the device slot, then attends them:
+    bit for bit vdx_rope3d on the whole tensors followed by vdx_attn_fwd on the
+    same blocks of rows (one block: the device vdx_attn_fwd_rope3d call)."""
+    from paper_2609_18077_gb300 import binding, workloads
+    import oracle
+    B, H, D = 2, 3, 128
+    grid, s0, dims, theta = (3, 6, 10), 9, (44, 42, 42), 1e4
+    S = s0 + grid[0] * grid[1] * grid[2] + 4
+    q, k, v = workloads.random_qkv(B, H, S, S, D, 4700 + r, 1.5)
+    scale = D ** -0.5
+    out, lse = binding.attn_fwd_rope3d_host(*(t.pin_memory() for t in (q, k, v)), grid, s0, dims, theta, True,
+                                            scale=scale, chunk_rows=r)
+    qr = binding.rope3d(q.cuda(), grid, s0, dims, theta, True).cpu()
+    kr = binding.rope3d(k.cuda(), grid, s0, dims, theta, True).cpu()
+    if r == 0:
+        o_dev, l_dev = binding.attn_fwd_rope3d(q.cuda(), k.cuda(), v.cuda(), grid, s0, dims, theta, True, scale=scale)
+        o_dev, l_dev = o_dev.cpu(), l_dev.cpu()   # library-chosen chunks: compared to the oracle below
+    else:
+        o_dev, l_dev = _device_chunks(qr, kr, v, scale, r)
+        assert torch.equal(out, o_dev)
+        assert torch.equal(lse, l_dev)
+    q_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(q), grid, s0, dims, theta, True)).to(torch.bfloat16)
+    k_ref = torch.from_numpy(oracle.rope3d(workloads.bf16_bits(k), grid, s0, dims, theta, True)).to(torch.bfloat16)
+    o_ref, lse_ref = run_oracle(q_ref, k_ref, v, scale)
+    compare(out, lse, o_ref, lse_ref)

@@ -195,3 +195,15 @@ def test_rope_attention_validates(lib):
     assert call(S=0) == 0                              # nothing to do
     assert f(g["q"] + 8, g["k"], g["v"], g["out"], g["lse"], 1, 1, 8, 128, 2, 2, 2, 0, 44, 42, 42, 1e4, 1, 0.1,
              None) == 3                                # q not 16-byte aligned
+
+
+def test_rope3d_host_validates(lib):
+    import torch
+    q = torch.zeros(1, 1, 8, 128, dtype=torch.bfloat16)
+    o = torch.zeros_like(q)
+    f = lib.vdx_attn_fwd_rope3d_host
+    a = (q.data_ptr(), q.data_ptr(), q.data_ptr(), o.data_ptr(), None, 1, 1, 8, 128)
+    assert f(*a, 2, 2, 2, 0, 45, 42, 42, 1e4, 1, 0.1, 0, None) == 1     # odd part
+    assert f(*a, 2, 2, 2, 0, 44, 42, 42, 0.0, 1, 0.1, 0, None) == 1     # theta
+    assert f(*a, 2, 2, 2, -1, 44, 42, 42, 1e4, 1, 0.1, 0, None) == 1    # s0
+    assert f(*a, 2, 2, 2, 0, 44, 42, 42, 1e4, 1, 0.1, -1, None) == 1    # chunk_rows
