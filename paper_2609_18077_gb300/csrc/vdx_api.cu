@@ -130,11 +130,11 @@ int device_ready(int *sms = nullptr)
     return st.status;
 }
 
-// Workspace of the split tail and of the segment key-tile lists, one per
-// (device, stream): calls on one stream
-// run in order, so they can share it; calls on different streams never do.
-// Allocated on the first call that needs it, grown when a later call needs
-// more (cudaFree waits for work still using the old one), kept until exit.
+// Library-owned device buffers, one per (device, stream, kind): calls on one
+// stream run in order, so they can share them; calls on different streams
+// never do.  Allocated on the first call that needs one, grown when a later
+// call needs more (cudaFree waits for work still using the old one), kept
+// until exit.
 struct Workspace {
     void *ptr = nullptr;
     size_t bytes = 0;
@@ -186,8 +186,9 @@ bool overlaps(const void *a, size_t na, const void *b, size_t nb)
     return x < y + nb && y < x + na;
 }
 
-// Per-problem-kind inputs: the valid key counts (MODE_VARLEN) or the
-// segment ids (MODE_SEG).
+// Per-problem-kind inputs: the valid key counts (MODE_VARLEN), the segment
+// ids (MODE_SEG) or the grid and window (MODE_WIN).  Device pointers for the
+// device calls; host pointers when handed to the host-buffer pipeline.
 struct KeyRule {
     int mode = vdx::MODE_DENSE;
     const int *kv_lens = nullptr;
