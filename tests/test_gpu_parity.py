@@ -1,6 +1,5 @@
 """CUDA path vs the fp64 oracle, element by element, on seeded inputs (GB300 only)."""
 import math
-import os
 
 import numpy as np
 import pytest

@@ -12,7 +12,7 @@ import math
 import pytest
 import torch
 
-from parity import check_case, compare, run_gpu, run_oracle
+from parity import compare, run_gpu, run_oracle
 
 from paper_2609_18077_gb300 import workloads
 

@@ -10,7 +10,6 @@ import subprocess
 import sys
 import tempfile
 
-import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 SOURCE = os.path.join(ROOT, "oracle", "oracle.c")

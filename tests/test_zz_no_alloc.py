@@ -11,7 +11,6 @@ that free device memory does not move while it runs.  It is collected last.
 import ctypes
 import math
 
-import numpy as np
 import pytest
 import torch
 
