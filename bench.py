@@ -5,16 +5,17 @@
 One step = one attention forward (one vdx_attn_fwd / vdx_attn_fwd_varlen /
 vdx_attn_fwd_segments / vdx_attn_fwd_win3d / vdx_attn_fwd_rope3d call) over
 the whole workload, inputs
-resident in HBM.  The default workload is the small-DiT 480p self-attention (B=1, H=12,
-D=128, S = 21*30*52 = 32760 tokens, logit std ~3).  FLOPs = 4*B*H*Sq*Skv*D
+resident in HBM.  The default workload is the largest single-GPU
+configuration, the large-DiT 720p self-attention (B=1, H=40, D=128,
+S = 21*45*80 = 75600 tokens).  FLOPs = 4*B*H*Sq*Skv*D
 (effective key counts for the padded-text workload; the (query, key) pairs
 of equal segment id for the joint text-video workload; the (query, key)
 pairs inside the windows for the windowed workload).
 
 Timing: W untimed warm-up steps, then K steps bracketed by a barrier and a
 device synchronisation, timed with CUDA events on the launching stream; the
-max over ranks is reported.  Inputs (Q, K, V, O: 403 MB) exceed the 129 MB
-L2, so no flush is inserted.  SM clocks are sampled with nvidia-smi during
+max over ranks is reported.  Inputs (large720's Q, K, V and O: 3.1 GB)
+exceed the 129 MB L2, so no flush is inserted.  SM clocks are sampled with nvidia-smi during
 the timed region.  A second timed pass ("e2e") starts from pinned host
 buffers: every step copies Q, K, V host->device, runs the kernel and copies
 O and LSE back.  Each step is one host-buffer call (vdx_attn_fwd_host, or its
@@ -24,7 +25,9 @@ chunks and overlaps the copies with the kernels.
 --impl reference times the fp64 CPU oracle (the only reference this
 method has) on a bounded row sample of the same workload.  Under torchrun
 (N > 1) each rank runs its own copy of the workload (independent problems:
-weak scaling, no collective on the data path).
+weak scaling, no collective on the data path).  --gpus N > 1 outside torchrun
+relaunches this script under torch.distributed.run with N processes; inside
+torchrun it must equal WORLD_SIZE.
 """
 from __future__ import annotations
 
@@ -428,16 +431,21 @@ def run_reference(args):
         timer.run()
     recs = [timer.run() for _ in range(args.steps)]
     value = statistics.median(r["value"] for r in recs)
-    ms_per_step = flops / (value * 1e12) * 1e3
+    # ms_per_step: the wall time of one timed step (one sample), as run; the
+    # full call at the sampled rate is reported beside it
+    ms_per_step = statistics.median(r["seconds"] for r in recs) * 1e3
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded N(0,1) bf16 tensors shaped like the workload; no dataset)",
-        "config": {"workload": wl.name, "B": wl.B, "H": wl.H, "Sq": wl.Sq, "Skv": wl.Skv, "D": wl.D,
-                   "flops_per_call": flops,
-                   "note": "each step times the oracle on a bounded row sample; ms_per_step is the "
-                           "full call extrapolated from the sampled rate"},
+        "config": {"workload": wl.name, "description": wl.description, "B": wl.B, "H": wl.H, "Sq": wl.Sq,
+                   "Skv": wl.Skv, "D": wl.D, "scale": wl.scale, "flops_per_call": flops,
+                   "parallelism": f"replicas x{world} (rank 0 times the oracle)",
+                   "note": "each step times the oracle on a bounded seeded row sample of the workload; "
+                           "ms_per_step is one such step; ms_full_call_extrapolated is the whole call at "
+                           "the sampled rate",
+                   "ms_full_call_extrapolated": round(flops / (value * 1e12) * 1e3, 1)},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": recs[-1]["cores"], "kind": "oracle",
                          "sample": recs[-1]["sample"] + " per step"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -449,7 +457,7 @@ def run_reference(args):
 def main():
     from paper_2609_18077_gb300 import workloads
     ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
-    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--gpus", type=int, default=None, help="GPUs (default: WORLD_SIZE under torchrun, else 1)")
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--workload", default=workloads.DEFAULT_WORKLOAD, choices=sorted(workloads.WORKLOADS))
@@ -457,6 +465,18 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     args = ap.parse_args()
+    if "WORLD_SIZE" not in os.environ and (args.gpus or 1) > 1:
+        # one process per GPU: relaunch under torchrun on this node
+        import socket
+        with socket.socket() as sock:
+            sock.bind(("127.0.0.1", 0))
+            port = sock.getsockname()[1]
+        cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", f"--nproc-per-node={args.gpus}",
+               "--master-addr", "127.0.0.1", "--master-port", str(port), os.path.abspath(__file__)] + sys.argv[1:]
+        sys.exit(subprocess.call(cmd))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if args.gpus is not None and args.gpus != world:
+        ap.error(f"--gpus {args.gpus} but WORLD_SIZE is {world}")
     if args.warmup < 3 and args.impl == "ours":
         print("note: fewer than 3 warm-up steps", file=sys.stderr)
     if args.impl == "reference":

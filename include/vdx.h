@@ -29,15 +29,18 @@
  *     library never frees or keeps them after the call returns.
  *   - Memory: when the last round of work units would leave most
  *     multiprocessors idle (dense calls only), the library splits those units
- *     along the keys and merges the parts through a device workspace of
- *     (tail units x parts x 2 x 128 x (D + 4)) fp32 values -- about 19 MB for
- *     B=1, H=12, S=32760, D=128.  Segment calls keep their key-tile lists in
- *     the same workspace: B x ceil(Sq/256) x ceil(Skv/128) x 4 bytes plus
- *     ranges (about 0.5 MB for B=2, S=45106).  The workspace belongs to the library, one per
- *     (device, stream): it is allocated by the first call that needs it, grown
- *     by a later call that needs more (that call waits for the device), and
- *     kept until the process exits.  Calls on the same stream share it in
- *     stream order; calls on different streams never share it.
+ *     along the keys and merges the parts through a device scratch of at most
+ *     (multiprocessors x 2 x 128 x (D + 4)) fp32 values plus counters -- about
+ *     20.6 MB on a 152-SM GB300.  It is allocated at that bound by the first
+ *     call on a stream that splits, so no later dense call on that stream
+ *     allocates or frees device memory.  Segment and window calls keep their
+ *     key-tile lists in a second buffer that grows with the problem
+ *     (B x ceil(Sq/256) x ceil(Skv/128) x 4 bytes plus ranges, about 0.5 MB
+ *     for B=2, S=45106); growing it frees the old one, which waits for the
+ *     device.  These buffers belong to the library, one set per (device,
+ *     stream): calls on the same stream share them in stream order, calls on
+ *     different streams never share them.  They are kept until
+ *     vdx_release(stream) or process exit.
  *   - q, k, v and out must be 16-byte aligned (TMA and vector stores); lse
  *     4-byte aligned.  out must not overlap q, k or v.
  *   - D must be 64 or 128.  B, H, Sq, Skv >= 0; B*H*Sq == 0 is a no-op.
@@ -62,7 +65,10 @@ typedef enum vdx_status {
     VDX_ERR_MISALIGNED = 3,  /* a pointer breaks the alignment rules above */
     VDX_ERR_CUDA = 4,        /* a CUDA runtime/driver call failed */
     VDX_ERR_DEVICE = 5,      /* the current device is not an sm_103 GPU */
-    VDX_ERR_TIMEOUT = 6      /* a bounded in-kernel wait expired (see vdx_check_device_error) */
+    VDX_ERR_TIMEOUT = 6,     /* a bounded in-kernel wait expired (see vdx_check_device_error) */
+    VDX_ERR_DRAIN = 7        /* a kernel that gave up could not confirm that its TMA loads or
+                                tensor-core operations had finished before it exited (see
+                                vdx_check_device_error); treat device memory as suspect */
 } vdx_status;
 
 /*
@@ -169,24 +175,27 @@ int vdx_attn_fwd_rope3d(const void *q, const void *k, const void *v, void *out, 
 /*
  * vdx_attn_fwd without any device allocation (the paper has no counterpart;
  * this is a library service).  Same arguments, results and errors as
- * vdx_attn_fwd, for callers that must not allocate device memory: code that
- * runs where cudaMalloc is not allowed or would stall the device (a stream
- * being captured into a graph, a serving loop whose memory is planned up
- * front, a process whose device memory belongs to another allocator).
+ * vdx_attn_fwd -- the outputs are bit for bit those of vdx_attn_fwd, which
+ * runs the same kernel with the same split -- for callers that cannot call
+ * cudaMalloc during the call: code that runs while a stream is being
+ * captured into a graph (an allocation there breaks the capture), a serving
+ * loop whose device memory is planned before it starts, a process whose
+ * device memory belongs to another allocator.
  *
- * Instead of the library's per-stream workspace, the split-tail scratch lives
+ * Instead of the library's per-stream scratch, the split-tail scratch lives
  * in a fixed 24 MiB array of device memory inside the library image, which
  * every GPU that loads the library holds until the process exits.  A call
  * whose scratch need exceeds 24 MiB returns VDX_ERR_UNSUPPORTED and launches
  * nothing (with at most one part per multiprocessor the need stays near
  * 21 MB at D = 128 on a 152-SM GB300).
  *
- * The first call on a device also looks up that array's device address
- * (once per device, the device being current); make that first call before
- * any stream capture.  Every call on a device shares the one array and it
- * keeps the previous call's contents: each call clears its counters itself,
- * on its stream, before the kernel.  Calls whose work overlaps on the GPU
- * (different streams, or threads without ordering) race on the array, so
+ * Arguments are checked exactly as vdx_attn_fwd checks them, before any CUDA
+ * call.  The first call on a device then looks up that array's device
+ * address (once per device, the device being current); make that first call
+ * before any stream capture.  Every call on a device shares the one array and
+ * it keeps the previous call's contents: each call clears its counters
+ * itself, on its stream, before the kernel.  Calls whose work overlaps on the
+ * GPU (different streams, or threads without ordering) race on the array, so
  * order them.  No cudaMalloc, cudaFree or allocating library routine is
  * called.
  */
@@ -265,14 +274,34 @@ int vdx_attn_fwd_win3d_host(const void *q, const void *k, const void *v, void *o
                             int B, int H, int F, int Hp, int Wp, int D, int kt, int kh, int kw,
                             int neighbourhood, float scale, long long chunk_rows, void *stream);
 
+/*
+ * Releases the device memory the library keeps for `stream` on the current
+ * device (a library service; the paper has no counterpart): the split-tail
+ * scratch and key-tile lists of the device calls, the turned q and k of
+ * vdx_attn_fwd_rope3d, and the host-buffer pipeline (its device slots,
+ * events and internal streams, and the scratch of its compute streams).
+ * Synchronises `stream` and the pipeline's streams first.  The next call on
+ * `stream` allocates again.  Call it only while no other thread enqueues work
+ * on `stream` through this library.  Returns VDX_OK (also when nothing was
+ * kept) or VDX_ERR_CUDA.
+ */
+int vdx_release(void *stream);
+
 /* Human-readable name of a vdx_status (static storage; never NULL). */
 const char *vdx_status_string(int status);
 
 /*
- * Synchronises `stream`, then reads and clears the library's device error
- * word on the current device.  Returns VDX_OK, VDX_ERR_TIMEOUT if a kernel
- * gave up on a bounded wait since the last check, or VDX_ERR_CUDA if the
- * synchronisation itself failed.
+ * Synchronises `stream`, then takes the library's device error word on the
+ * current device: reads and zeroes it in one atomic exchange, so a bit a
+ * kernel sets meanwhile is reported by this check or the next, never lost.
+ * The word is per device, shared by every stream: a kernel on another stream
+ * that gave up since the last check is reported here too.  Returns VDX_OK;
+ * VDX_ERR_TIMEOUT if a kernel gave up on a bounded wait (its work stopped
+ * cleanly: every copy and tensor-core operation it issued had finished before
+ * it exited); VDX_ERR_DRAIN if a kernel could not confirm that (the GPU broke
+ * a completion guarantee; treat device memory as suspect); VDX_ERR_CUDA if
+ * the synchronisation or the read failed.  Checks from several threads are
+ * serialised.
  */
 int vdx_check_device_error(void *stream);
 

@@ -6,5 +6,5 @@ it.  The library is loaded on first use and its absence is an error.
 """
 from .binding import (VdxError, attn_fwd, attn_fwd_host, attn_fwd_rope3d, attn_fwd_rope3d_host,  # noqa: F401
                       attn_fwd_segments, attn_fwd_segments_host, attn_fwd_varlen, attn_fwd_win3d,
-                      attn_fwd_win3d_host, check_device_error, load, rope3d, selftest_wait_timeout,
+                      attn_fwd_win3d_host, check_device_error, load, release, rope3d, selftest_wait_timeout,
                       status_string, version)

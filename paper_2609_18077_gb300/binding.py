@@ -24,6 +24,7 @@ VDX_ERR_MISALIGNED = 3
 VDX_ERR_CUDA = 4
 VDX_ERR_DEVICE = 5
 VDX_ERR_TIMEOUT = 6
+VDX_ERR_DRAIN = 7
 
 # Every symbol include/vdx.h declares, with its ctypes signature.
 _P = ctypes.c_void_p
@@ -44,6 +45,7 @@ SIGNATURES = {
                                                                          ctypes.c_longlong, _P]),
     "vdx_status_string": (ctypes.c_char_p, [_I]),
     "vdx_check_device_error": (_I, [_P]),
+    "vdx_release": (_I, [_P]),
     "vdx_selftest_wait_timeout": (_I, [_I, _P]),
     "vdx_version": (_I, []),
 }
@@ -90,6 +92,15 @@ def check_device_error(device=None) -> int:
     device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
     with torch.cuda.device(device):
         return int(load().vdx_check_device_error(_stream_handle(device)))
+
+
+def release(device=None) -> None:
+    """Free the device memory the library keeps for the current stream of `device`."""
+    device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    with torch.cuda.device(device):
+        st = int(load().vdx_release(_stream_handle(device)))
+    if st != VDX_OK:
+        raise VdxError(st, "vdx_release")
 
 
 def selftest_wait_timeout(limit_us: int, device=None) -> int:

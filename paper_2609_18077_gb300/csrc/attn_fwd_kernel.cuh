@@ -59,8 +59,12 @@
 // boxes instead (stages_out below).
 //
 // Every wait is bounded (globaltimer); on expiry the CTA records
-// VDX_ERR_TIMEOUT in the device error word, skips the rest of its work, frees
-// its tensor memory and returns.
+// VDX_ERR_TIMEOUT in the device error word and skips the rest of its work.
+// Before it exits, the producer waits for every TMA load it issued to land
+// and the issuer for every tensor-core operation it issued to retire (both
+// complete by themselves, so these waits cannot be stranded by another
+// warp); only then is tensor memory freed and the CTA's shared memory, which
+// those loads write and whose barriers they signal, given up.
 #pragma once
 
 #include <cuda.h>
@@ -81,9 +85,19 @@ constexpr int MODE_WIN = 3;      // the keys inside the query's 3D window (S = F
 // Modes that visit key tiles from a list and may mask a row's every key so far.
 __host__ __device__ constexpr bool listed(int mode) { return mode == MODE_SEG || mode == MODE_WIN; }
 
-// Device error word: bit 0 = a bounded wait expired.  Read and cleared by
-// vdx_check_device_error.
+// Device error word, one per device, shared by every launch; taken (read and
+// zeroed in one atomic exchange) by vdx_check_device_error.
+//   bit 0: a bounded wait expired and the CTA gave up its work;
+//   bit 1: the issuer's final wait for its tensor-core operations expired, so
+//          tensor memory was released with operations possibly in flight;
+//   bit 2: a TMA load issued by the producer had not landed when the CTA was
+//          about to exit (its wait for the load expired).
+// Bits 1 and 2 mean the GPU broke a completion guarantee; bit 0 alone means
+// the work stopped cleanly.
 __device__ unsigned int g_error_word;
+constexpr unsigned ERR_WAIT_EXPIRED = 1u;
+constexpr unsigned ERR_MMA_DRAIN = 2u;
+constexpr unsigned ERR_LOADS_IN_FLIGHT = 4u;
 
 constexpr int BM = 128;          // query rows per tile (= TMEM lanes)
 constexpr int BN = 128;          // keys per tile
@@ -197,11 +211,25 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, vola
                 return false;
             if (ptx::globaltimer_ns() - t0 > limit_ns) {
                 *abort_flag = 1;
-                atomicOr(&g_error_word, 1u);
+                atomicOr(&g_error_word, ERR_WAIT_EXPIRED);
                 return false;
             }
         }
     }
+}
+
+// Wait for a phase that completes by itself -- TMA bytes landing on a barrier
+// whose arrivals were all made, or tensor-core operations retiring -- whatever
+// the abort flag says.  Bounded all the same; false if the limit expired.
+__device__ __forceinline__ bool wait_landed(uint32_t bar, uint32_t parity, uint64_t limit_ns)
+{
+    if (ptx::mbar_try_wait(bar, parity))
+        return true;
+    const uint64_t t0 = ptx::globaltimer_ns();
+    while (!ptx::mbar_try_wait(bar, parity))
+        if (ptx::globaltimer_ns() - t0 > limit_ns)
+            return false;
+    return true;
 }
 
 __device__ __forceinline__ float ex2(float x)
@@ -561,8 +589,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     return i;
             }
         };
-        int g = 0;
-        int fixes = 0;
+        int g = 0;          // stages armed so far
+        int fixes = 0;      // B_FIX phases completed
+        bool fix_pending = false;   // a B_FIX phase armed but not seen complete
+        uint32_t q_armed = 0;       // bit b: Q barrier b armed at least once
+        uint32_t q_parity = 0;      // bit b: parity of Q barrier b's last armed phase
         bool ok = true;
         // load stage g: V tile (vbh, vj) if vj >= 0, K tile (kbh, kj) if kj >= 0.
         // MODE_SEG: the V tile's list entry goes to the stage's slot before the
@@ -572,10 +603,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         auto stage = [&](int vbh, int vj, int v_valid, int kbh, int kj, uint32_t ventry) -> bool {
             const int st = g % L::NSTAGE;
             const int rnd = g / L::NSTAGE;
-            ++g;
             if (rnd > 0 &&
                 !__all_sync(0xffffffffu, wait_bounded(bar(L::B_EMPTY + st), (rnd - 1) & 1, abort_flag, limit)))
                 return false;
+            ++g;
             const uint32_t vdst = sbase + L::KV_OFF + (2 * st) * L::TILE_BYTES;
             const uint32_t kdst = vdst + L::TILE_BYTES;
             const bool has_v = vj >= 0, has_k = kj >= 0;
@@ -597,8 +628,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                              kj * BN, kbh);
                     }
                 }
-                if (!__all_sync(0xffffffffu, wait_bounded(bar(L::B_FIX), fixes & 1, abort_flag, limit)))
+                fix_pending = true;
+                if (!__all_sync(0xffffffffu, wait_bounded(bar(L::B_FIX), fixes & 1, abort_flag, limit))) {
+                    // Give the stage its one arrival, so that its phase completes
+                    // once the K bytes land and the drain below can see them land.
+                    if (lane == 0)
+                        ptx::mbar_arrive(bar(L::B_FULL + st));
                     return false;
+                }
+                fix_pending = false;
                 ++fixes;
                 const int per_half = (BN - v_valid) * 8;   // 16-byte chunks per 64-column block
                 uint8_t *slot_ptr = sm + L::KV_OFF + (2 * st) * L::TILE_BYTES;
@@ -667,6 +705,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         ptx::tma_load_3d(sbase + L::Q_OFF + (2 * qb + t) * L::TILE_BYTES + h * L::HALF_BYTES,
                                          &tmap_q, bar(L::B_Q + 2 * qb + t), h * 64, (w.qp * 2 + t) * BM, w.bh);
                 }
+                if (ok) {
+                    const uint32_t bit = 1u << (2 * qb + t);
+                    q_armed |= bit;
+                    q_parity = (q_parity & ~bit) | (((iq / QBUF) & 1) ? bit : 0u);
+                }
             }
             if (!ok)
                 break;
@@ -694,6 +737,27 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             }
             i = ni;
         }
+        // Every TMA load above completes on a barrier in this CTA's shared
+        // memory, and none may still be in flight when the CTA exits: after an
+        // abort the consumers stop waiting for them, so the producer waits for
+        // the last armed phase of every barrier it loads to (all its arrivals
+        // were made, so the phase completes by itself once the bytes land).
+        // Without an abort every such phase was consumed and these checks pass
+        // at once.
+        if (lane == 0) {
+            bool landed = true;
+            for (int st = 0; st < L::NSTAGE; ++st)
+                if (g > st)
+                    landed &= wait_landed(bar(L::B_FULL + st), ((g - 1 - st) / L::NSTAGE) & 1, limit);
+            for (int b = 0; b < 2 * QBUF; ++b)
+                if ((q_armed >> b) & 1u)
+                    landed &= wait_landed(bar(L::B_Q + b), (q_parity >> b) & 1u, limit);
+            if (fix_pending)
+                landed &= wait_landed(bar(L::B_FIX), fixes & 1, limit);
+            if (!landed)
+                atomicOr(&g_error_word, ERR_LOADS_IN_FLIGHT);
+        }
+        __syncwarp();
     } else if (warp == MMA_WARP) {
         // ------------------------------------------------------------ tcgen05 issuer
         if (lane == 0) {
@@ -778,15 +842,16 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 g += n;
                 ++iq;
             }
-            // Retire every MMA this thread issued before TMEM is released.
+            // Retire every MMA this thread issued (and with them the arrivals
+            // their commits make on this CTA's barriers) before TMEM is
+            // released.  They need nothing from other warps, so they retire
+            // within microseconds.  Should this wait still expire, bit 1 of
+            // the error word records it and tensor memory is released all the
+            // same: a CTA that exits holding tensor memory would leave every
+            // later allocation on its multiprocessor waiting forever.
             ptx::mma_commit(bar(L::B_DRAIN));
-            const uint64_t t0 = ptx::globaltimer_ns();
-            while (!ptx::mbar_try_wait(bar(L::B_DRAIN), 0)) {
-                if (ptx::globaltimer_ns() - t0 > limit) {
-                    atomicOr(&g_error_word, 1u);
-                    break;
-                }
-            }
+            if (!wait_landed(bar(L::B_DRAIN), 0, limit))
+                atomicOr(&g_error_word, ERR_MMA_DRAIN);
         }
         __syncwarp();
     } else {
@@ -1074,6 +1139,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         ptx::tmem_dealloc(tmem, TMEM_COLS);
     }
 }
+
+// Takes the device error word: zeroes it and leaves its old value in
+// g_error_taken, in one atomic exchange, so no bit set meanwhile is lost.
+__device__ unsigned int g_error_taken;
+__global__ void error_word_take_kernel() { g_error_taken = atomicExch(&g_error_word, 0u); }
 
 // Failure-detection self-test: one thread waits on a barrier nothing arrives on.
 __global__ void wait_timeout_selftest_kernel(uint64_t limit_ns)

@@ -106,8 +106,8 @@ __device__ __forceinline__ bool pair_turn(const RopeParams &p, int pair, long lo
 }
 
 // One adjacent bf16 pair (x_a in the low half) turned by (c, sn).  Rounded
-// products and a fused add, spelled out so that every caller (this kernel and
-// the attention kernel's fused Q rotation) gets the same bits.
+// products and a fused add, spelled out so that the vectorised kernel and the
+// one-pair-per-thread kernel give the same bits.
 __device__ __forceinline__ uint32_t rotate_pair(uint32_t word, float c, float sn)
 {
     const __nv_bfloat162 e = *reinterpret_cast<const __nv_bfloat162 *>(&word);

@@ -132,20 +132,23 @@ int device_ready(int *sms = nullptr)
 
 // Library-owned device buffers, one per (device, stream, kind): calls on one
 // stream run in order, so they can share them; calls on different streams
-// never do.  Allocated on the first call that needs one, grown when a later
-// call needs more (cudaFree waits for work still using the old one), kept
-// until exit.
+// never do.  Allocated on the first call that needs one and kept until
+// vdx_release or exit.  The split-tail scratch is allocated at its bound
+// (one part per multiprocessor at D = 128), so once a stream has one no later
+// dense call allocates or frees anything; the kinds that scale with the
+// problem grow when a call needs more (cudaFree waits for work still using
+// the old buffer).
 struct Workspace {
     void *ptr = nullptr;
     size_t bytes = 0;
 };
-// kind: WS_TAIL (split tail, key-tile lists) or WS_ROPE_K / WS_ROPE_Q (the
-// turned K and Q of vdx_attn_fwd_rope3d).
-enum { WS_TAIL = 0, WS_ROPE_K = 1, WS_ROPE_Q = 2 };
+// kind: WS_SPLIT (split tail), WS_LISTS (key-tile lists of segment and window
+// calls), WS_ROPE_K / WS_ROPE_Q (the turned K and Q of vdx_attn_fwd_rope3d).
+enum { WS_SPLIT = 0, WS_LISTS = 1, WS_ROPE_K = 2, WS_ROPE_Q = 3, WS_KINDS = 4 };
 std::mutex g_ws_mutex;
 std::map<std::tuple<int, cudaStream_t, int>, Workspace> g_ws;
 
-int workspace(int dev, cudaStream_t stream, size_t bytes, void **out, int kind = WS_TAIL)
+int workspace(int dev, cudaStream_t stream, size_t bytes, void **out, int kind)
 {
     std::lock_guard<std::mutex> lock(g_ws_mutex);
     Workspace &w = g_ws[std::make_tuple(dev, stream, kind)];
@@ -162,7 +165,37 @@ int workspace(int dev, cudaStream_t stream, size_t bytes, void **out, int kind =
     return VDX_OK;
 }
 
+// Frees the workspaces of (dev, stream); the caller has synchronised stream.
+int release_workspaces(int dev, cudaStream_t stream)
+{
+    std::lock_guard<std::mutex> lock(g_ws_mutex);
+    int st = VDX_OK;
+    for (int kind = 0; kind < WS_KINDS; ++kind) {
+        auto it = g_ws.find(std::make_tuple(dev, stream, kind));
+        if (it == g_ws.end())
+            continue;
+        if (it->second.ptr && cudaFree(it->second.ptr) != cudaSuccess)
+            st = VDX_ERR_CUDA;
+        g_ws.erase(it);
+    }
+    return st;
+}
+
 size_t round_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Split-tail scratch of `cells` (tail units x parts, at most one per CTA)
+// at head dim D: unnormalised O, then the row statistics, then the counters.
+struct SplitLayout {
+    size_t o_bytes, st_bytes, cnt_bytes;
+    size_t total() const { return o_bytes + st_bytes + cnt_bytes; }
+};
+SplitLayout split_layout(size_t cells, size_t tail, int D)
+{
+    return {round_up(cells * 2 * vdx::BM * D * 4, 256), round_up(cells * 2 * vdx::BM * 16, 256),
+            round_up(tail * 4, 256)};
+}
+// Its bound on a device with `sms` multiprocessors: tail x parts <= grid <= sms.
+size_t split_bound_bytes(int sms) { return split_layout(sms, sms, 128).total(); }
 
 // [B*H, rows, D] bf16 tensor as a 3-D TMA map with 64 x box_rows x 1 boxes, 128-B swizzle.
 int make_map(CUtensorMap *map, const void *base, long long rows, long long bh, int D, int box_rows = vdx::BM)
@@ -197,17 +230,15 @@ struct KeyRule {
     vdx::WinGrid win{};   // MODE_WIN
 };
 
-// fixed_scratch / fixed_bytes: when set, the split-tail workspace is taken
-// from that fixed device region instead of the library's allocation.
-int attn_launch(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
-                int D, const KeyRule &rule, float scale, void *stream, void *fixed_scratch = nullptr,
-                size_t fixed_bytes = 0)
+// Checks the arguments of an attention call without any CUDA call.  VDX_OK
+// with *empty = true means there is nothing to launch.
+int attn_check(const void *q, const void *k, const void *v, const void *out, const float *lse, int B, int H, int Sq,
+               int Skv, int D, const KeyRule &rule, float scale, bool *empty)
 {
     const bool varlen = rule.mode == vdx::MODE_VARLEN;
     const bool seg = rule.mode == vdx::MODE_SEG;
-    const bool win = rule.mode == vdx::MODE_WIN;
     const int *kv_lens = rule.kv_lens;
-    // ---- validation (no CUDA calls)
+    *empty = false;
     if (!q || !k || !v || !out || (varlen && !kv_lens) || (seg && (!rule.q_seg || !rule.kv_seg)))
         return VDX_ERR_INVALID_ARG;
     if (B < 0 || H < 0 || Sq < 0 || Skv < 0)
@@ -220,8 +251,10 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         (kv_lens && !aligned(kv_lens, 4)) || (seg && (!aligned(rule.q_seg, 4) || !aligned(rule.kv_seg, 4))))
         return VDX_ERR_MISALIGNED;
     const long long bh = static_cast<long long>(B) * H;
-    if (bh == 0 || Sq == 0)
+    if (bh == 0 || Sq == 0) {
+        *empty = true;
         return VDX_OK;
+    }
     if (bh > INT_MAX)
         return VDX_ERR_INVALID_ARG;
     const long long q_tiles = (Sq + vdx::BM - 1) / vdx::BM;
@@ -233,6 +266,27 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     if (overlaps(out, q_bytes, q, q_bytes) || (kv_bytes && (overlaps(out, q_bytes, k, kv_bytes) ||
                                                            overlaps(out, q_bytes, v, kv_bytes))))
         return VDX_ERR_INVALID_ARG;
+    return VDX_OK;
+}
+
+// fixed_scratch / fixed_bytes: when set, the split-tail workspace is taken
+// from that fixed device region instead of the library's allocation.
+int attn_launch(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
+                int D, const KeyRule &rule, float scale, void *stream, void *fixed_scratch = nullptr,
+                size_t fixed_bytes = 0)
+{
+    const bool varlen = rule.mode == vdx::MODE_VARLEN;
+    const bool seg = rule.mode == vdx::MODE_SEG;
+    const bool win = rule.mode == vdx::MODE_WIN;
+    const int *kv_lens = rule.kv_lens;
+    // ---- validation (no CUDA calls)
+    bool empty = false;
+    int chk = attn_check(q, k, v, out, lse, B, H, Sq, Skv, D, rule, scale, &empty);
+    if (chk != VDX_OK || empty)
+        return chk;
+    const long long bh = static_cast<long long>(B) * H;
+    const long long q_tiles = (Sq + vdx::BM - 1) / vdx::BM;
+    const long long q_pairs = (q_tiles + 1) / 2;
 
     // ---- device set-up
     int sms = 0;
@@ -288,26 +342,27 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     if (parts > n_kv)
         parts = n_kv;
     if (parts >= 2) {
-        const size_t o_bytes = round_up(static_cast<size_t>(tail) * parts * 2 * vdx::BM * D * 4, 256);
-        const size_t st_bytes = round_up(static_cast<size_t>(tail) * parts * 2 * vdx::BM * 16, 256);
-        const size_t cnt_bytes = round_up(static_cast<size_t>(tail) * 4, 256);
+        const SplitLayout sl = split_layout(static_cast<size_t>(tail) * parts, tail, D);
         int dev = 0;
         void *ws = nullptr;
-        if (cudaGetDevice(&dev) != cudaSuccess)
-            return VDX_ERR_CUDA;
         if (fixed_scratch) {
-            if (o_bytes + st_bytes + cnt_bytes > fixed_bytes)
+            if (sl.total() > fixed_bytes)
                 return VDX_ERR_UNSUPPORTED;
             ws = fixed_scratch;
-        } else if ((st = workspace(dev, s, o_bytes + st_bytes + cnt_bytes, &ws)) != VDX_OK) {
-            return st;
+        } else {
+            if (cudaGetDevice(&dev) != cudaSuccess)
+                return VDX_ERR_CUDA;
+            size_t need = split_bound_bytes(sms);
+            need = need > sl.total() ? need : sl.total();
+            if ((st = workspace(dev, s, need, &ws, WS_SPLIT)) != VDX_OK)
+                return st;
         }
         p.split_parts = parts;
         p.full_rounds = full_rounds;
         p.tail_units = tail;
         p.ws_o = static_cast<float *>(ws);
-        p.ws_stats = reinterpret_cast<float *>(static_cast<char *>(ws) + o_bytes);
-        p.ws_count = reinterpret_cast<int *>(static_cast<char *>(ws) + o_bytes + st_bytes);
+        p.ws_stats = reinterpret_cast<float *>(static_cast<char *>(ws) + sl.o_bytes);
+        p.ws_count = reinterpret_cast<int *>(static_cast<char *>(ws) + sl.o_bytes + sl.st_bytes);
         if (cudaMemsetAsync(p.ws_count, 0, static_cast<size_t>(tail) * 4, s) != cudaSuccess)
             return VDX_ERR_CUDA;
     }
@@ -325,7 +380,7 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         void *ws = nullptr;
         if (cudaGetDevice(&dev) != cudaSuccess)
             return VDX_ERR_CUDA;
-        if ((st = workspace(dev, s, kr_bytes + qr_bytes + list_bytes + cnt_bytes, &ws)) != VDX_OK)
+        if ((st = workspace(dev, s, kr_bytes + qr_bytes + list_bytes + cnt_bytes, &ws, WS_LISTS)) != VDX_OK)
             return st;
         char *base = static_cast<char *>(ws);
         int2 *krange = reinterpret_cast<int2 *>(base);
@@ -353,7 +408,7 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         void *ws = nullptr;
         if (cudaGetDevice(&dev) != cudaSuccess)
             return VDX_ERR_CUDA;
-        if ((st = workspace(dev, s, list_bytes + cnt_bytes, &ws)) != VDX_OK)
+        if ((st = workspace(dev, s, list_bytes + cnt_bytes, &ws, WS_LISTS)) != VDX_OK)
             return st;
         uint32_t *tlist = static_cast<uint32_t *>(ws);
         int *tcount = reinterpret_cast<int *>(static_cast<char *>(ws) + list_bytes);
@@ -891,13 +946,13 @@ extern "C" {
 int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq,
                          int Skv, int D, float scale, void *stream)
 {
-    // Argument checks first, exactly as vdx_attn_fwd does them, so a bad call
-    // touches no CUDA state; then the fixed scratch's device address.
-    if (!q || !k || !v || !out || B < 0 || H < 0 || Sq < 0 || Skv < 0 || (D != 64 && D != 128) ||
-        !std::isfinite(scale))
-        return VDX_ERR_INVALID_ARG;
-    if (static_cast<long long>(B) * H == 0 || Sq == 0)
-        return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, KeyRule{}, scale, stream);
+    // The argument checks of vdx_attn_fwd come first, so that a bad call
+    // returns the same status and touches no CUDA state; then the fixed
+    // scratch's device address.
+    bool empty = false;
+    const int chk = attn_check(q, k, v, out, lse, B, H, Sq, Skv, D, KeyRule{}, scale, &empty);
+    if (chk != VDX_OK || empty)
+        return chk;
     void *scratch = nullptr;
     const int st = noalloc_scratch(&scratch);
     if (st != VDX_OK)
@@ -905,7 +960,6 @@ int vdx_attn_fwd_noalloc(const void *q, const void *k, const void *v, void *out,
     return attn_launch(q, k, v, out, lse, B, H, Sq, Skv, D, KeyRule{}, scale, stream, scratch,
                        kNoAllocScratchBytes);
 }
-
 
 int vdx_attn_fwd(const void *q, const void *k, const void *v, void *out, float *lse, int B, int H, int Sq, int Skv,
                  int D, float scale, void *stream)
@@ -1060,24 +1114,75 @@ const char *vdx_status_string(int status)
     case VDX_ERR_CUDA: return "VDX_ERR_CUDA: CUDA call failed";
     case VDX_ERR_DEVICE: return "VDX_ERR_DEVICE: current device is not sm_103";
     case VDX_ERR_TIMEOUT: return "VDX_ERR_TIMEOUT: bounded in-kernel wait expired";
+    case VDX_ERR_DRAIN:
+        return "VDX_ERR_DRAIN: a kernel that gave up could not confirm its copies or tensor-core work had finished";
     default: return "unknown vdx status";
     }
 }
 
 int vdx_check_device_error(void *stream)
 {
-    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess)
         return VDX_ERR_CUDA;
+    const int st = device_ready();
+    if (st != VDX_OK)
+        return st;
+    // One check at a time takes the word (through one snapshot variable).
+    static std::mutex take_mutex;
+    std::lock_guard<std::mutex> lock(take_mutex);
     unsigned int word = 0;
-    if (cudaMemcpyFromSymbol(&word, vdx::g_error_word, sizeof word) != cudaSuccess)
+    vdx::error_word_take_kernel<<<1, 1, 0, s>>>();
+    if (cudaGetLastError() != cudaSuccess ||
+        cudaMemcpyFromSymbolAsync(&word, vdx::g_error_taken, sizeof word, 0, cudaMemcpyDeviceToHost, s) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
         return VDX_ERR_CUDA;
-    if (word != 0) {
-        const unsigned int zero = 0;
-        if (cudaMemcpyToSymbol(vdx::g_error_word, &zero, sizeof zero) != cudaSuccess)
-            return VDX_ERR_CUDA;
-        return VDX_ERR_TIMEOUT;
+    if (word & (vdx::ERR_MMA_DRAIN | vdx::ERR_LOADS_IN_FLIGHT))
+        return VDX_ERR_DRAIN;
+    return word ? VDX_ERR_TIMEOUT : VDX_OK;
+}
+
+int vdx_release(void *stream)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (cudaStreamSynchronize(s) != cudaSuccess)
+        return VDX_ERR_CUDA;
+    int st = release_workspaces(dev, s);
+    // The host-buffer pipeline of (dev, stream): its slots, events, streams,
+    // and the workspaces of its compute streams.
+    std::unique_lock<std::mutex> lock(g_pipes_mutex);
+    auto it = g_pipes.find({dev, s});
+    if (it == g_pipes.end())
+        return st;
+    HostPipe &pp = it->second;
+    {
+        std::lock_guard<std::mutex> pipe_lock(pp.mutex);
+        if (pp.ready) {
+            for (cudaStream_t own : {pp.up, pp.run[0], pp.run[1], pp.down})
+                if (cudaStreamSynchronize(own) != cudaSuccess)
+                    st = VDX_ERR_CUDA;
+            for (cudaStream_t own : {pp.run[0], pp.run[1]})
+                if (release_workspaces(dev, own) != VDX_OK)
+                    st = VDX_ERR_CUDA;
+        }
+        if (pp.buf && cudaFree(pp.buf) != cudaSuccess)
+            st = VDX_ERR_CUDA;
+        for (int i = 0; i < kHostSlots; ++i)
+            for (cudaEvent_t e : {pp.h2d[i], pp.comp[i], pp.d2h[i]})
+                if (e && cudaEventDestroy(e) != cudaSuccess)
+                    st = VDX_ERR_CUDA;
+        if (pp.start && cudaEventDestroy(pp.start) != cudaSuccess)
+            st = VDX_ERR_CUDA;
+        for (cudaStream_t own : {pp.up, pp.run[0], pp.run[1], pp.down})
+            if (own && cudaStreamDestroy(own) != cudaSuccess)
+                st = VDX_ERR_CUDA;
     }
-    return VDX_OK;
+    g_pipes.erase(it);
+    return st;
 }
 
 int vdx_selftest_wait_timeout(int limit_us, void *stream)

@@ -144,8 +144,9 @@ WORKLOADS = {
                     "tokens, padded text masked by segment ids, CFG batch 2, D=64"),
 }
 
-# The bench's default workload: the small-DiT 480p self-attention.
-DEFAULT_WORKLOAD = "small480"
+# The bench's default workload: the largest single-GPU configuration, the
+# large-DiT 720p self-attention (B=1, H=40, D=128, S = 21*45*80 = 75600).
+DEFAULT_WORKLOAD = "large720"
 
 
 def _spawn(seed: int, n: int = 4):

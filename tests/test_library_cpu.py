@@ -35,7 +35,7 @@ def test_exports_every_declared_symbol(lib):
 def test_version_and_status(lib):
     from paper_2609_18077_gb300 import binding
     assert binding.version() == 10000
-    for s in range(7):
+    for s in range(8):
         assert binding.status_string(s).startswith("VDX_")
     assert binding.status_string(99) == "unknown vdx status"
 
@@ -60,6 +60,22 @@ def call(lib, **kw):
 ])
 def test_validation(lib, kw, status):
     assert call(lib, **kw) == status
+
+
+@pytest.mark.parametrize("kw,status", [
+    (dict(q=None), 1), (dict(out=None), 1), (dict(D=96), 1), (dict(B=-1), 1), (dict(scale=float("nan")), 1),
+    (dict(q=A + 8), 3), (dict(out=4 * A + 2), 3), (dict(lse=5 * A + 2), 3),
+    (dict(out=A), 1),                     # out overlaps q
+    (dict(B=0), 0), (dict(Sq=0), 0),
+])
+def test_noalloc_validation_matches(lib, kw, status):
+    """vdx_attn_fwd_noalloc rejects a bad call exactly as vdx_attn_fwd does,
+    before any CUDA call (on this CPU-only machine a CUDA call would fail with
+    VDX_ERR_CUDA instead)."""
+    a = {**GOOD, **kw}
+    args = (a["q"], a["k"], a["v"], a["out"], a["lse"], a["B"], a["H"], a["Sq"], a["Skv"], a["D"], a["scale"], None)
+    assert lib.vdx_attn_fwd_noalloc(*args) == status
+    assert lib.vdx_attn_fwd(*args) == status
 
 
 def test_varlen_requires_lengths(lib):

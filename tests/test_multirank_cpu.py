@@ -52,8 +52,8 @@ def test_max_over_ranks_single():
 @pytest.mark.parametrize("rank", [0, 1])
 def test_reference_arm_prints_on_rank0_only(rank):
     env = {**os.environ, "RANK": str(rank), "WORLD_SIZE": "2", "LOCAL_RANK": str(rank), "OMP_NUM_THREADS": "2"}
-    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--workload", "tiny",
-                        "--steps", "2", "--warmup", "1", "--cpu-seconds", "0.5"],
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--gpus", "2", "--impl", "reference",
+                        "--workload", "tiny", "--steps", "2", "--warmup", "1", "--cpu-seconds", "0.5"],
                        capture_output=True, text=True, env=env, timeout=600)
     assert r.returncode == 0, r.stderr
     lines = [ln for ln in r.stdout.splitlines() if ln.strip()]
@@ -64,3 +64,12 @@ def test_reference_arm_prints_on_rank0_only(rank):
         d = json.loads(lines[0])
         assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["unit"] == "TFLOP/s"
         assert d["cpu_baseline"]["kind"] == "oracle" and d["e2e"]["h2d_bytes_per_step"] == 0
+        # one step is one bounded sample: its measured time, not the full call's
+        assert d["ms_per_step"] < 60e3 and d["config"]["ms_full_call_extrapolated"] > 0
+
+
+def test_gpus_must_match_world_size():
+    env = {**os.environ, "RANK": "0", "WORLD_SIZE": "2", "LOCAL_RANK": "0"}
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--gpus", "4", "--impl", "reference",
+                        "--workload", "tiny"], capture_output=True, text=True, env=env, timeout=600)
+    assert r.returncode != 0 and "WORLD_SIZE" in r.stderr
