@@ -36,6 +36,7 @@ def test_no_allocation_after_setup_and_release():
     for extra, seed in ((2, 31), (5, 32)):
         q, k, v = (t.cuda() for t in workloads.random_qkv(1, sms + extra, 256, 2000, D, seed=seed, logit_gain=1.3))
         cases.append((q, k, v, torch.empty_like(q), torch.empty(q.shape[:3], dtype=torch.float32, device="cuda")))
+    first = [(torch.empty_like(o), torch.empty_like(l)) for *_, o, l in cases]   # copies of the first results
     side = torch.cuda.Stream()
     side.wait_stream(torch.cuda.current_stream())
     with torch.cuda.stream(side):
@@ -48,7 +49,10 @@ def test_no_allocation_after_setup_and_release():
         free1 = _free()
         assert binding.check_device_error(torch.device("cuda", 0)) == binding.VDX_OK
         assert free1 == free0, f"dense calls after set-up changed free memory by {free0 - free1} bytes"
-        first = [(o.clone(), l.clone()) for *_, o, l in cases]
+        for (*_, o, l), (o0, l0) in zip(cases, first):
+            o0.copy_(o)
+            l0.copy_(l)
+        assert _free() == free1
         binding.release()
         free2 = _free()
         assert free2 > free1, "vdx_release freed nothing"
