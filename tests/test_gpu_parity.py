@@ -63,6 +63,68 @@ def test_varlen(B, H, Sq, Skv, D, lens):
     check_case(B, H, Sq, Skv, D, 1 / math.sqrt(D), seed=300 + Sq + Skv, kv_lens=np.array(lens, np.int32))
 
 
+# Text cross-attention (padded text keys, per-sample lengths): lengths at
+# every key-tile border (0, 1, 127/128/129, 255/256/257, 383/384/385,
+# 511/512), short Skv_max, a single query row, and more work units than
+# multiprocessors so that every persistent CTA walks several (b, h).
+CROSS_EDGES = [0, 1, 127, 128, 129, 255, 256, 257, 300, 383, 384, 385, 511, 512]
+CROSS = [
+    # B, H, Sq, Skv_max, D, lens
+    (len(CROSS_EDGES), 2, 300, 512, 128, CROSS_EDGES),
+    (len(CROSS_EDGES), 2, 300, 512, 64, CROSS_EDGES),
+    (3, 2, 129, 200, 128, [200, 57, 0]),
+    (2, 3, 1, 256, 64, [256, 100]),
+    (4, 40, 640, 512, 128, [223, 215, 512, 300]),
+    (2, 48, 384, 512, 64, [0, 171]),
+]
+
+
+@pytest.mark.parametrize("B,H,Sq,Skv,D,lens", CROSS)
+def test_text_cross_attention(B, H, Sq, Skv, D, lens):
+    check_case(B, H, Sq, Skv, D, 1 / math.sqrt(D), seed=600 + B * H + Sq, gain=1.5,
+               kv_lens=np.array(lens, np.int32))
+
+
+@pytest.mark.parametrize("smul,gain", [(-1.0, 1.5), (0.0, 1.0), (4.0, 3.0)])
+def test_text_cross_attention_scales(smul, gain):
+    """Negative and zero logit scales, and logits spread wide enough that a
+    later key tile's maximum moves past the lazy-rescale threshold."""
+    lens = np.array([512, 300, 257, 40], np.int32)
+    check_case(4, 3, 260, 512, 128, smul / math.sqrt(128), seed=700, gain=gain, kv_lens=lens)
+
+
+def test_text_cross_attention_canaries_and_determinism():
+    """The varlen instance's TMA stores of O stay inside out (ragged Sq: the
+    last tile is clipped), LSE inside lse; two calls give the same bits."""
+    from paper_2609_18077_gb300 import binding, workloads
+    B, H, Sq, Skv, D = 3, 5, 200, 512, 128
+    lens = np.array([512, 129, 0], np.int32)
+    q, k, v = workloads.random_qkv(B, H, Sq, Skv, D, seed=11)
+    k, v = workloads.pad_invalid_keys(k, v, lens)
+    q, k, v = q.cuda(), k.cuda(), v.cuda()
+    ld = torch.from_numpy(lens).cuda()
+    pad = 4096
+    obuf = torch.full((pad + B * H * Sq * D + pad,), float("nan"), dtype=torch.bfloat16, device="cuda")
+    lbuf = torch.full((pad + B * H * Sq + pad,), float("nan"), dtype=torch.float32, device="cuda")
+    out = obuf[pad:pad + B * H * Sq * D].view(B, H, Sq, D)
+    lse = lbuf[pad:pad + B * H * Sq].view(B, H, Sq)
+    binding.attn_fwd_varlen(q, k, v, ld, scale=D ** -0.5, out=out, lse=lse)
+    assert binding.check_device_error() == binding.VDX_OK
+    assert torch.isnan(obuf[:pad]).all() and torch.isnan(obuf[-pad:]).all()
+    assert torch.isnan(lbuf[:pad]).all() and torch.isnan(lbuf[-pad:]).all()
+    assert torch.isfinite(out).all()
+    assert torch.isneginf(lse[2]).all() and torch.isfinite(lse[:2]).all()
+    o2, l2 = binding.attn_fwd_varlen(q, k, v, ld, scale=D ** -0.5)
+    assert torch.equal(out.view(torch.int16), o2.view(torch.int16)) and torch.equal(lse, l2)
+
+
+def test_varlen_long_text_many_units():
+    """Long padded key sequences with mixed lengths over many units (key
+    tiles skipped past each sample's length)."""
+    lens = np.array([0, 600, 1, 513, 129, 0, 256, 599], np.int32)
+    check_case(8, 20, 257, 600, 128, 128 ** -0.5, seed=502, kv_lens=lens)
+
+
 def test_tiny_workload_full():
     from paper_2609_18077_gb300 import workloads
     w = workloads.generate("tiny")
