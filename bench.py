@@ -165,7 +165,7 @@ def run_ours(args):
     mode = "seg" if segs is not None else ("varlen" if lens is not None else "dense")
     if wl.window is not None:
         mode = "win"
-        launches_per_step = 2     # key-tile lists, then the attention
+        launches_per_step = 1     # the attention (key boxes follow from each unit's index: no lists)
     rope = wl.rope
     if rope is not None:
         # the step turns Q and K (two RoPE launches), then attends

@@ -11,9 +11,10 @@
 // query i attend key j iff their segment ids match: each unit visits only the
 // key tiles of its list (segment_tiles.cuh) and compares ids element by
 // element only on the tiles the list marks.  The window instance (windowed 3D
-// attention, appendix Table 4's VAE decoder) walks per query-tile-pair lists
-// of the key tiles inside the unit's window box (window_tiles.cuh) and masks
-// keys outside each row's window.
+// attention, appendix Table 4's VAE decoder) takes its query tiles as 3-D
+// bricks of the token grid and walks a regular grid of 3-D key boxes over the
+// union of the unit's windows (window_tiles.cuh), through 5-D tensor maps,
+// masking keys outside each row's window.
 //
 // Work unit: one (b*h, pair of 128-row query tiles).  The grid is persistent:
 // one CTA per SM walks the units u = blockIdx.x, blockIdx.x + gridDim.x, ...
@@ -466,10 +467,14 @@ __device__ __forceinline__ Item unit_item(const AttnParams &p, const SegParams &
         w.kv_valid = len < 0 ? 0 : (len > p.Skv ? p.Skv : len);
     }
     w.n_kv = (w.kv_valid + BN - 1) / BN;
-    if (listed(MODE)) {
-        const int pair = MODE == MODE_WIN ? w.qp : (w.bh / p.H) * p.q_pairs + w.qp;
+    if (MODE == MODE_SEG) {
+        const int pair = (w.bh / p.H) * p.q_pairs + w.qp;
         w.n_kv = __ldg(sp.tcount + pair);
         w.list_off = pair * sp.n_kt;
+    }
+    if (MODE == MODE_WIN) {
+        const WinUnit u = win_unit(sp.win, w.qp);   // key boxes over the unit's window union
+        w.n_kv = u.nbt * u.nbh * u.nbw;
     }
     w.j0 = 0;
     w.j1 = w.n_kv;
@@ -508,13 +513,64 @@ __device__ __forceinline__ Item item_at(const AttnParams &p, const SegParams &sp
 }
 
 // List entry of position r of item w: in MODE_SEG the key tile and its mask
-// bits (segment_tiles.cuh); otherwise the key tile r itself.
+// bits (segment_tiles.cuh); otherwise r itself (the key tile, or in MODE_WIN
+// the key box).
 template <int MODE>
 __device__ __forceinline__ uint32_t tile_entry(const SegParams &sp, const Item &w, int r)
 {
-    if (listed(MODE))
+    if (MODE == MODE_SEG)
         return __ldg(sp.tlist + w.list_off + r);
     return static_cast<uint32_t>(r);
+}
+
+// Where a K or V tile (or, in MODE_WIN, a key box) sits in its tensor map:
+// (row, b*h) of the 3-D map, or (w, h, t, b*h) of the 5-D one.
+struct TileAt {
+    int bh;
+    int c0, c1, c2;
+};
+
+template <int MODE>
+__device__ __forceinline__ TileAt tile_at(const SegParams &sp, const Item &w, int j)
+{
+    TileAt a;
+    a.bh = w.bh;
+    if (MODE == MODE_WIN) {
+        const WinUnit u = win_unit(sp.win, w.qp);
+        win_box(sp.win, u, j, a.c2, a.c1, a.c0);
+    } else {
+        a.c0 = j * BN;
+        a.c1 = a.c2 = 0;
+    }
+    return a;
+}
+
+// One 64-column half (x = 0 or 64) of a tile, through the map's dimensionality.
+template <int MODE>
+__device__ __forceinline__ void tma_tile(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, const TileAt &a)
+{
+    if (MODE == MODE_WIN)
+        ptx::tma_load_5d(dst, map, bar, x, a.c0, a.c1, a.c2, a.bh);
+    else
+        ptx::tma_load_3d(dst, map, bar, x, a.c0, a.bh);
+}
+
+// Query tile t of item w: its 3-D tile (row) or, in MODE_WIN, its brick.
+template <int MODE>
+__device__ __forceinline__ TileAt q_tile_at(const SegParams &sp, const Item &w, int t)
+{
+    TileAt a;
+    a.bh = w.bh;
+    if (MODE == MODE_WIN) {
+        const WinUnit u = win_unit(sp.win, w.qp);
+        a.c0 = u.w0;
+        a.c1 = u.h0;
+        a.c2 = u.t0 + (t << sp.win.qlt);
+    } else {
+        a.c0 = (w.qp * 2 + t) * BM;
+        a.c1 = a.c2 = 0;
+    }
+    return a;
 }
 
 template <int D, int MODE, int QBUF, int NSTAGE>
@@ -595,12 +651,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         uint32_t q_armed = 0;       // bit b: Q barrier b armed at least once
         uint32_t q_parity = 0;      // bit b: parity of Q barrier b's last armed phase
         bool ok = true;
-        // load stage g: V tile (vbh, vj) if vj >= 0, K tile (kbh, kj) if kj >= 0.
-        // MODE_SEG: the V tile's list entry goes to the stage's slot before the
-        // full barrier is armed (its arrive releases the slot to the softmax,
-        // which reads it after its wait on that barrier; the slot is rewritten
-        // only after the stage is released, i.e. after that read).
-        auto stage = [&](int vbh, int vj, int v_valid, int kbh, int kj, uint32_t ventry) -> bool {
+        // load stage g: V tile va if has_v, K tile ka if has_k.
+        // Listed modes: the V tile's list entry (MODE_WIN: the key box's
+        // origin) goes to the stage's slot before the full barrier is armed
+        // (its arrive releases the slot to the softmax, which reads it after
+        // its wait on that barrier; the slot is rewritten only after the stage
+        // is released, i.e. after that read).
+        auto stage = [&](const TileAt &va, bool has_v, int v_valid, const TileAt &ka, bool has_k,
+                         uint32_t ventry) -> bool {
             const int st = g % L::NSTAGE;
             const int rnd = g / L::NSTAGE;
             if (rnd > 0 &&
@@ -609,7 +667,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             ++g;
             const uint32_t vdst = sbase + L::KV_OFF + (2 * st) * L::TILE_BYTES;
             const uint32_t kdst = vdst + L::TILE_BYTES;
-            const bool has_v = vj >= 0, has_k = kj >= 0;
             const bool fix = MODE == MODE_VARLEN && has_v && v_valid < BN;
             if (fix) {
                 // A padded sample's last V tile: rows past the valid length may
@@ -620,12 +677,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 if (lane == 0) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_FIX), L::TILE_BYTES);
                     for (int h = 0; h < D / 64; ++h)
-                        ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FIX), h * 64, vj * BN, vbh);
+                        tma_tile<MODE>(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FIX), h * 64, va);
                     if (has_k) {
                         ptx::mbar_expect_tx(bar(L::B_FULL + st), L::TILE_BYTES);
                         for (int h = 0; h < D / 64; ++h)
-                            ptx::tma_load_3d(kdst + h * L::HALF_BYTES, &tmap_k, bar(L::B_FULL + st), h * 64,
-                                             kj * BN, kbh);
+                            tma_tile<MODE>(kdst + h * L::HALF_BYTES, &tmap_k, bar(L::B_FULL + st), h * 64, ka);
                     }
                 }
                 fix_pending = true;
@@ -655,21 +711,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     volatile uint32_t *slot = reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF) + 4 * st;
                     slot[0] = ventry;
                     if (MODE == MODE_WIN) {
-                        int t0, h0, w0;
-                        grid_pos(sp.win, vj * BN, t0, h0, w0);
-                        slot[1] = static_cast<uint32_t>(t0) | (static_cast<uint32_t>(h0) << 16);
-                        slot[2] = static_cast<uint32_t>(w0);
+                        // the key box's origin (t | h << 16, w)
+                        slot[1] = static_cast<uint32_t>(va.c2) | (static_cast<uint32_t>(va.c1) << 16);
+                        slot[2] = static_cast<uint32_t>(va.c0);
                     }
                 }
                 if (bytes) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_FULL + st), bytes);
                     for (int h = 0; h < D / 64; ++h) {
                         if (has_v && !fix)
-                            ptx::tma_load_3d(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FULL + st), h * 64,
-                                             vj * BN, vbh);
+                            tma_tile<MODE>(vdst + h * L::HALF_BYTES, &tmap_v, bar(L::B_FULL + st), h * 64, va);
                         if (has_k)
-                            ptx::tma_load_3d(kdst + h * L::HALF_BYTES, &tmap_k, bar(L::B_FULL + st), h * 64,
-                                             kj * BN, kbh);
+                            tma_tile<MODE>(kdst + h * L::HALF_BYTES, &tmap_k, bar(L::B_FULL + st), h * 64, ka);
                     }
                 } else {
                     ptx::mbar_arrive(bar(L::B_FULL + st));
@@ -687,7 +740,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         }
         if (i >= 0) {
             const Item w = item_at<MODE>(p, sp, cta, i);
-            ok = stage(0, -1, BN, w.bh, static_cast<int>(tile_entry<MODE>(sp, w, w.j0) & SEG_TILE_BITS), 0u);
+            const TileAt none{0, 0, 0, 0};
+            ok = stage(none, false, BN, tile_at<MODE>(sp, w, static_cast<int>(tile_entry<MODE>(sp, w, w.j0) &
+                                                                              SEG_TILE_BITS)),
+                       true, 0u);
         }
         for (int iq = 0; ok && i >= 0; ++iq) {
             const Item w = item_at<MODE>(p, sp, cta, i);
@@ -701,9 +757,10 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                                                               abort_flag, limit));
                 if (ok && lane == 0) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_Q + 2 * qb + t), L::TILE_BYTES);
+                    const TileAt qa = q_tile_at<MODE>(sp, w, t);
                     for (int h = 0; h < D / 64; ++h)
-                        ptx::tma_load_3d(sbase + L::Q_OFF + (2 * qb + t) * L::TILE_BYTES + h * L::HALF_BYTES,
-                                         &tmap_q, bar(L::B_Q + 2 * qb + t), h * 64, (w.qp * 2 + t) * BM, w.bh);
+                        tma_tile<MODE>(sbase + L::Q_OFF + (2 * qb + t) * L::TILE_BYTES + h * L::HALF_BYTES, &tmap_q,
+                                       bar(L::B_Q + 2 * qb + t), h * 64, qa);
                 }
                 if (ok) {
                     const uint32_t bit = 1u << (2 * qb + t);
@@ -721,18 +778,25 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             // ran; start bringing them to L2 now so that load is short (a hint:
             // nothing waits for it).
             if (lane == 0 && nw.ok)
-                for (int t = 0; t < 2; ++t)
-                    for (int h = 0; h < D / 64; ++h)
-                        ptx::tma_prefetch_3d(&tmap_q, h * 64, (nw.qp * 2 + t) * BM, nw.bh);
+                for (int t = 0; t < 2; ++t) {
+                    const TileAt qa = q_tile_at<MODE>(sp, nw, t);
+                    for (int h = 0; h < D / 64; ++h) {
+                        if (MODE == MODE_WIN)
+                            ptx::tma_prefetch_5d(&tmap_q, h * 64, qa.c0, qa.c1, qa.c2, qa.bh);
+                        else
+                            ptx::tma_prefetch_3d(&tmap_q, h * 64, qa.c0, qa.bh);
+                    }
+                }
             uint32_t ve = tile_entry<MODE>(sp, w, w.j0);
             for (int j = w.j0; ok && j < w.j1; ++j) {
                 const bool last = j + 1 == w.j1;
-                const int kbh = last ? (nw.ok ? nw.bh : 0) : w.bh;
                 // MODE_SEG: the list entry is read before the stage's empty wait
                 const uint32_t ke = last ? (nw.ok ? tile_entry<MODE>(sp, nw, nw.j0) : 0u) : tile_entry<MODE>(sp, w, j + 1);
-                const int kj = (last && !nw.ok) ? -1 : static_cast<int>(ke & SEG_TILE_BITS);
+                const bool has_k = !(last && !nw.ok);
+                const int kj = static_cast<int>(ke & SEG_TILE_BITS);
                 const int vj = static_cast<int>(ve & SEG_TILE_BITS);
-                ok = stage(w.bh, vj, w.kv_valid - vj * BN, kbh, kj, ve);
+                const TileAt ka = has_k ? tile_at<MODE>(sp, last ? nw : w, kj) : TileAt{0, 0, 0, 0};
+                ok = stage(tile_at<MODE>(sp, w, vj), true, w.kv_valid - vj * BN, ka, has_k, ve);
                 ve = ke;
             }
             i = ni;
@@ -873,8 +937,21 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             const Item w = item_at<MODE>(p, sp, cta, i);
             if (!w.ok)
                 break;
-            const int q_row = (w.qp * 2 + t) * BM + row;
-            const bool store = q_row < p.Sq;
+            // This row's query: its token index q_row (stores and LSE) and, in
+            // MODE_WIN, its window (one packed axis per word) for the whole unit;
+            // a brick row outside the grid stores nothing and sees no key.
+            int q_row = (w.qp * 2 + t) * BM + row;
+            bool store = q_row < p.Sq;
+            uint32_t win_t = 0, win_h = 0, win_w = 0;
+            if (MODE == MODE_WIN) {
+                const WinUnit u = win_unit(sp.win, w.qp);
+                const int pw = u.w0 + (row & ((1 << sp.win.qlw) - 1));
+                const int ph = u.h0 + ((row >> sp.win.qlw) & ((1 << sp.win.qlh) - 1));
+                const int pt = u.t0 + (t << sp.win.qlt) + (row >> (sp.win.qlw + sp.win.qlh));
+                store = pt < sp.win.F && ph < sp.win.Hp && pw < sp.win.Wp;
+                q_row = store ? (pt * sp.win.Hp + ph) * sp.win.Wp + pw : 0;
+                packed_window(sp.win, pt, ph, pw, win_t, win_h, win_w);
+            }
             __nv_bfloat16 *orow = p.out + (static_cast<size_t>(w.bh) * p.Sq + (store ? q_row : 0)) * D;
             if (w.j1 == w.j0) {
                 if (store) {
@@ -889,10 +966,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
             float m_used = -INFINITY;
             float l_exact = 0.f;   // sum of the fp32 weights: the log-sum-exp
             float l_resid = 0.f;   // sum over tiles of r - p for each tile's largest weight
-            // MODE_WIN: this row's window, one packed axis per word, for the whole unit
-            uint32_t win_t = 0, win_h = 0, win_w = 0;
-            if (MODE == MODE_WIN)
-                packed_window(sp.win, store ? q_row : 0, win_t, win_h, win_w);
             for (int j = w.j0; j < w.j1; ++j, ++sc) {
                 if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_S + t), sc & 1, abort_flag, limit))))
                     break;
@@ -902,22 +975,15 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 // that wait comes first here; the row's 128-key window mask is
                 // then built while the logits are not yet in registers.
                 uint32_t wmask[4] = {0u, 0u, 0u, 0u};
-                bool win_mask = false;
-                int kt_win = j;
                 if (MODE == MODE_WIN) {
                     if (!(ok = __all_sync(0xffffffffu, wait_bounded(bar(L::B_FULL + gj % L::NSTAGE),
                                                                     (gj / L::NSTAGE) & 1, abort_flag, limit))))
                         break;
                     const volatile uint32_t *slot =
                         reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF) + 4 * (gj % L::NSTAGE);
-                    const uint32_t entry = slot[0];
-                    kt_win = static_cast<int>(entry & SEG_TILE_BITS);
-                    win_mask = (entry >> (SEG_MASK_SHIFT + t)) & 1u;
-                    if (win_mask) {
-                        const uint32_t th = slot[1];
-                        window_mask(sp.win, p.Sq, win_t, win_h, win_w, kt_win, static_cast<int>(th & 0xFFFFu),
-                                    static_cast<int>(th >> 16), static_cast<int>(slot[2]), wmask);
-                    }
+                    const uint32_t th = slot[1];
+                    window_mask(sp.win, win_t, win_h, win_w, static_cast<int>(th & 0xFFFFu),
+                                static_cast<int>(th >> 16), static_cast<int>(slot[2]), wmask);
                 }
                 uint32_t s[4][32];
 #pragma unroll
@@ -933,7 +999,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 }
                 ptx::tmem_wait_ld();
 
-                int kt = MODE == MODE_WIN ? kt_win : j;   // key tile
+                int kt = j;   // key tile
                 bool seg_mask = false;
                 if (MODE == MODE_SEG) {
                     // the stage's list entry, published with its full barrier
@@ -942,7 +1008,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                     seg_mask = (entry >> (SEG_MASK_SHIFT + t)) & 1u;
                 }
                 const int valid = w.kv_valid - kt * BN;
-                if (valid < BN) {
+                if (MODE != MODE_WIN && valid < BN) {
                     // Ragged last tile: keys past the end (or past the sample's
                     // text length, whatever their bits) become -inf logits
                     // after scaling, i.e. weight exactly 0.  scale_log2 is never
@@ -973,8 +1039,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         s[c >> 5][c & 31] = kid == my_seg ? s[c >> 5][c & 31] : pad;
                     }
                 }
-                if (MODE == MODE_WIN && win_mask) {
-                    // keys outside this row's window get the masked logit
+                if (MODE == MODE_WIN) {
+                    // keys outside this row's window (or the grid) get the masked logit
                     const uint32_t pad = neg_scale ? 0x7F800000u : 0xFF800000u;
 #pragma unroll
                     for (int c = 0; c < BN; ++c)

@@ -142,8 +142,8 @@ struct Workspace {
     void *ptr = nullptr;
     size_t bytes = 0;
 };
-// kind: WS_SPLIT (split tail), WS_LISTS (key-tile lists of segment and window
-// calls), WS_ROPE_K / WS_ROPE_Q (the turned K and Q of vdx_attn_fwd_rope3d).
+// kind: WS_SPLIT (split tail), WS_LISTS (key-tile lists of segment calls),
+// WS_ROPE_K / WS_ROPE_Q (the turned K and Q of vdx_attn_fwd_rope3d).
 enum { WS_SPLIT = 0, WS_LISTS = 1, WS_ROPE_K = 2, WS_ROPE_Q = 3, WS_KINDS = 4 };
 std::mutex g_ws_mutex;
 std::map<std::tuple<int, cudaStream_t, int>, Workspace> g_ws;
@@ -209,6 +209,73 @@ int make_map(CUtensorMap *map, const void *base, long long rows, long long bh, i
                                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? VDX_OK : VDX_ERR_CUDA;
+}
+
+// [B*H, F, Hp, Wp, D] bf16 tensor (a token grid per (b, h)) as a 5-D TMA map
+// (D, Wp, Hp, F, B*H) with 64 x bw x bh x bt x 1 boxes: one box is a 3-D
+// brick of bt*bh*bw tokens, landing as that many 128-byte rows (w fastest)
+// in the 128-byte swizzle of the 3-D maps.
+int make_map5(CUtensorMap *map, const void *base, const vdx::WinGrid &g, long long bh, int D, int lt, int lh, int lw)
+{
+    const cuuint64_t dims[5] = {static_cast<cuuint64_t>(D), static_cast<cuuint64_t>(g.Wp),
+                                static_cast<cuuint64_t>(g.Hp), static_cast<cuuint64_t>(g.F),
+                                static_cast<cuuint64_t>(bh)};
+    const cuuint64_t row = static_cast<cuuint64_t>(D) * 2;
+    const cuuint64_t strides[4] = {row, row * g.Wp, row * g.Wp * g.Hp, row * g.Wp * g.Hp * g.F};
+    const cuuint32_t box[5] = {64, 1u << lw, 1u << lh, 1u << lt, 1};
+    const cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    const CUresult r = encode_fn()(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(base), dims, strides,
+                                   box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? VDX_OK : VDX_ERR_CUDA;
+}
+
+// Key boxes of side 2^lk along one axis of length L, summed over the units
+// along it (each covering `span` consecutive positions from span * j).
+long long axis_boxes(int L, int k, int neighbourhood, int span, int lk)
+{
+    long long n = 0;
+    for (int p0 = 0; p0 < L; p0 += span) {
+        int lo, hi;
+        vdx::axis_union(p0, p0 + span - 1, L, k, neighbourhood, lo, hi);
+        n += (hi - lo + (1 << lk)) >> lk;
+    }
+    return n;
+}
+
+// Brick and key-box shapes of a windowed problem: among all query bricks of
+// 128 tokens (a unit is two of them stacked in t) and all key boxes of 128
+// tokens whose t-slices hold at most 32 keys, the pair with the fewest key
+// steps in all, each unit also counted as two steps for its start and
+// epilogue.  The step count is a product of per-axis sums, so the search is
+// cheap.  Fills the shape fields of g; returns the units per (b, h).
+long long choose_win_shapes(vdx::WinGrid &g)
+{
+    double best = -1.0;
+    long long best_units = 0;
+    for (int qt = 0; qt <= 7; ++qt)
+        for (int qh = 0; qt + qh <= 7; ++qh) {
+            const int qw = 7 - qt - qh;
+            const long long nut = (g.F + (2 << qt) - 1) / (2 << qt);
+            const long long nuh = (g.Hp + (1 << qh) - 1) >> qh, nuw = (g.Wp + (1 << qw) - 1) >> qw;
+            const long long units = nut * nuh * nuw;
+            for (int kt = 2; kt <= 7; ++kt)
+                for (int kh = 0; kt + kh <= 7; ++kh) {
+                    const int kw = 7 - kt - kh;
+                    const double steps = static_cast<double>(axis_boxes(g.F, g.kt, g.neighbourhood, 2 << qt, kt)) *
+                                         static_cast<double>(axis_boxes(g.Hp, g.kh, g.neighbourhood, 1 << qh, kh)) *
+                                         static_cast<double>(axis_boxes(g.Wp, g.kw, g.neighbourhood, 1 << qw, kw));
+                    const double cost = steps + 2.0 * static_cast<double>(units);
+                    if (best < 0 || cost < best) {
+                        best = cost;
+                        best_units = units;
+                        g.qlt = qt, g.qlh = qh, g.qlw = qw;
+                        g.klt = kt, g.klh = kh, g.klw = kw;
+                        g.nuh = static_cast<int>(nuh), g.nuw = static_cast<int>(nuw);
+                    }
+                }
+        }
+    return best_units;
 }
 
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
@@ -286,7 +353,14 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         return chk;
     const long long bh = static_cast<long long>(B) * H;
     const long long q_tiles = (Sq + vdx::BM - 1) / vdx::BM;
-    const long long q_pairs = (q_tiles + 1) / 2;
+    long long q_pairs = (q_tiles + 1) / 2;
+    vdx::WinGrid wg = rule.win;
+    if (win) {
+        // query bricks and key boxes (window_tiles.cuh); a unit is two bricks
+        q_pairs = choose_win_shapes(wg);
+        if (bh * q_pairs > INT_MAX)
+            return VDX_ERR_UNSUPPORTED;
+    }
 
     // ---- device set-up
     int sms = 0;
@@ -296,9 +370,15 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
 
     CUtensorMap mq, mk, mv, mo;
     const long long kv_rows = Skv > 0 ? Skv : 1;   // never loaded when Skv == 0
-    if ((st = make_map(&mq, q, Sq, bh, D)) != VDX_OK || (st = make_map(&mk, k, kv_rows, bh, D)) != VDX_OK ||
-        (st = make_map(&mv, v, kv_rows, bh, D)) != VDX_OK)
+    if (win) {
+        if ((st = make_map5(&mq, q, wg, bh, D, wg.qlt, wg.qlh, wg.qlw)) != VDX_OK ||
+            (st = make_map5(&mk, k, wg, bh, D, wg.klt, wg.klh, wg.klw)) != VDX_OK ||
+            (st = make_map5(&mv, v, wg, bh, D, wg.klt, wg.klh, wg.klw)) != VDX_OK)
+            return st;
+    } else if ((st = make_map(&mq, q, Sq, bh, D)) != VDX_OK || (st = make_map(&mk, k, kv_rows, bh, D)) != VDX_OK ||
+               (st = make_map(&mv, v, kv_rows, bh, D)) != VDX_OK) {
         return st;
+    }
     // The output map (32-row boxes, one per softmax warp) serves the instance
     // that stores O through TMA; the others never read it.
     std::memset(&mo, 0, sizeof(mo));
@@ -400,27 +480,8 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         sp.tcount = tcount;
         sp.n_kt = n_kv;
     }
-    if (win) {
-        // Key-tile lists per query-tile pair, shared by every (b, h).
-        const size_t list_bytes = round_up(static_cast<size_t>(q_pairs) * n_kv * 4, 256);
-        const size_t cnt_bytes = round_up(static_cast<size_t>(q_pairs) * 4, 256);
-        int dev = 0;
-        void *ws = nullptr;
-        if (cudaGetDevice(&dev) != cudaSuccess)
-            return VDX_ERR_CUDA;
-        if ((st = workspace(dev, s, list_bytes + cnt_bytes, &ws, WS_LISTS)) != VDX_OK)
-            return st;
-        uint32_t *tlist = static_cast<uint32_t *>(ws);
-        int *tcount = reinterpret_cast<int *>(static_cast<char *>(ws) + list_bytes);
-        vdx::win_tile_lists_kernel<<<static_cast<unsigned>((q_pairs + 7) / 8), 256, 0, s>>>(
-            rule.win, Sq, static_cast<int>(q_pairs), n_kv, tlist, tcount);
-        if (cudaGetLastError() != cudaSuccess)
-            return VDX_ERR_CUDA;
-        sp.tlist = tlist;
-        sp.tcount = tcount;
-        sp.n_kt = n_kv;
-        sp.win = rule.win;
-    }
+    if (win)
+        sp.win = wg;   // no lists: each unit's key boxes follow from its index
     using vdx::MODE_DENSE;
     using vdx::MODE_SEG;
     using vdx::MODE_VARLEN;

@@ -1,4 +1,4 @@
-// Key-tile lists of windowed 3D attention, for sm_103a.
+// Geometry of windowed 3D attention, for sm_103a.
 //
 // What it serves (vidax paper, appendix Table 4: the LTX-2.5 VAE decoder's 3D
 // neighbourhood attention, an 11 x 11 x 11 window).  The S = F*Hp*Wp tokens of
@@ -8,22 +8,23 @@
 //     neighbourhood: [lo, min(lo + k, L) - 1], lo = clamp(p - k/2, 0, max(L - k, 0))
 //                    (shifted inward at the border);
 //     truncated:     [max(p - k/2, 0), min(p + k/2, L - 1)].
-// Both bounds are non-decreasing in p.
+// Both bounds are non-decreasing in p, so the windows of a run of positions
+// [p0, p1] cover exactly [lo(p0), hi(p1)].
 //
-// One small launch before the attention kernel builds, for every pair of
-// 128-row query tiles (the attention kernel's unit; the same for every batch
-// and head), the ordered list of key tiles holding at least one key inside
-// the unit's window box -- per axis, the union of the windows of the unit's
-// smallest and largest coordinate, a superset of every query's window -- and
-// marks per query tile whether the key tile needs the element-wise window
-// test (it does not when all its keys lie inside the intersection of that
-// query tile's windows).
+// Tiles are 3-D boxes of the grid, not runs of the raster order.  A query
+// tile is a brick of qbt x qbh x qbw = 128 tokens (TMA loads it through a
+// 5-D tensor map (D, Wp, Hp, F, B*H) as 128 rows, w fastest); a unit is two
+// bricks stacked in t.  The union of the windows of a unit's queries is then
+// one box, and the unit's key tiles are a regular grid of kbt x kbh x kbw =
+// 128-token boxes laid over it from its low corner: no key-tile list is
+// needed, each box's origin follows from its index.  Boxes reaching past the
+// union or the grid hold keys that no query of the unit attends (TMA fills
+// positions outside the grid with zeros); the per-row mask removes them.
+// The host chooses both box shapes to minimise the key boxes visited; the
+// pattern of one t-slice of a key box (kbh x kbw bits) fits one 32-bit word.
 #pragma once
 
-#include <climits>
 #include <cstdint>
-
-#include "segment_tiles.cuh"
 
 namespace vdx {
 
@@ -31,128 +32,72 @@ struct WinGrid {
     int F, Hp, Wp;       // grid; S = F * Hp * Wp
     int kt, kh, kw;      // odd window sizes
     int neighbourhood;   // 1: shifted inward at the border; 0: truncated
+    // log2 of the query brick and key box sides (t, h, w), each triple summing to 7
+    int qlt, qlh, qlw;
+    int klt, klh, klw;
+    int nuh, nuw;        // units along h and w (the unit index is (jt * nuh + jh) * nuw + jw)
 };
 
-__device__ __forceinline__ void axis_window(int p, int L, int k, int neighbourhood, int &lo, int &hi)
+__host__ __device__ __forceinline__ void axis_window(int p, int L, int k, int neighbourhood, int &lo, int &hi)
 {
     if (neighbourhood) {
         const int last = L - k > 0 ? L - k : 0;
-        lo = min(max(p - k / 2, 0), last);
-        hi = min(lo + k, L) - 1;
+        lo = p - k / 2;
+        lo = lo < 0 ? 0 : (lo > last ? last : lo);
+        hi = (lo + k < L ? lo + k : L) - 1;
     } else {
-        lo = max(p - k / 2, 0);
-        hi = min(p + k / 2, L - 1);
+        lo = p - k / 2 < 0 ? 0 : p - k / 2;
+        hi = p + k / 2 < L - 1 ? p + k / 2 : L - 1;
     }
 }
 
-// Coordinates of token index i.
-__device__ __forceinline__ void grid_pos(const WinGrid &g, int i, int &t, int &h, int &w)
+// Union of the windows of positions [p0, p1] (clipped to the axis) along one axis.
+__host__ __device__ __forceinline__ void axis_union(int p0, int p1, int L, int k, int neighbourhood, int &lo, int &hi)
 {
-    const int hw = g.Hp * g.Wp;
-    t = i / hw;
-    const int r = i - t * hw;
-    h = r / g.Wp;
-    w = r - h * g.Wp;
+    int a, b;
+    p1 = p1 < L - 1 ? p1 : L - 1;
+    axis_window(p0, L, k, neighbourhood, lo, a);
+    axis_window(p1, L, k, neighbourhood, b, hi);
 }
 
-// One warp per query-tile pair qp: tlist[qp * n_kt + r] for r < tcount[qp].
-__global__ void __launch_bounds__(256) win_tile_lists_kernel(const WinGrid g, int S, int q_pairs, int n_kt,
-                                                             uint32_t *__restrict__ tlist, int *__restrict__ tcount)
+// A unit's geometry: the origin of its first query brick and the union box
+// of its queries' windows, with the key-box counts along each axis.
+struct WinUnit {
+    int t0, h0, w0;            // first brick's origin (the second is qbt further in t)
+    int ut, uh, uw;            // union box low corner
+    int nbt, nbh, nbw;         // key boxes per axis
+};
+
+__host__ __device__ __forceinline__ WinUnit win_unit(const WinGrid &g, int qp)
 {
-    const int qp = static_cast<int>((static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x) >> 5);
-    const int lane = threadIdx.x & 31;
-    if (qp >= q_pairs)
-        return;
-    // per query tile t: the smallest and largest t, h, w among its rows
-    int mn[2][3], mx[2][3];
-#pragma unroll
-    for (int q = 0; q < 2; ++q) {
-#pragma unroll
-        for (int a = 0; a < 3; ++a) {
-            mn[q][a] = INT_MAX;
-            mx[q][a] = INT_MIN;
-        }
-        for (int e = lane; e < 128; e += 32) {
-            const int i = (2 * qp + q) * 128 + e;
-            if (i < S) {
-                int c[3];
-                grid_pos(g, i, c[0], c[1], c[2]);
-#pragma unroll
-                for (int a = 0; a < 3; ++a) {
-                    mn[q][a] = min(mn[q][a], c[a]);
-                    mx[q][a] = max(mx[q][a], c[a]);
-                }
-            }
-        }
-#pragma unroll
-        for (int a = 0; a < 3; ++a)
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                mn[q][a] = min(mn[q][a], __shfl_xor_sync(0xFFFFFFFFu, mn[q][a], o));
-                mx[q][a] = max(mx[q][a], __shfl_xor_sync(0xFFFFFFFFu, mx[q][a], o));
-            }
-    }
-    const int len[3] = {g.F, g.Hp, g.Wp};
-    const int ks[3] = {g.kt, g.kh, g.kw};
-    // union box of both tiles and, per tile, the intersection of its windows
-    int ulo[3], uhi[3], ilo[2][3], ihi[2][3];
-    bool has[2];
-#pragma unroll
-    for (int q = 0; q < 2; ++q)
-        has[q] = mn[q][0] != INT_MAX;
-#pragma unroll
-    for (int a = 0; a < 3; ++a) {
-        ulo[a] = INT_MAX;
-        uhi[a] = INT_MIN;
-#pragma unroll
-        for (int q = 0; q < 2; ++q) {
-            ilo[q][a] = 0;
-            ihi[q][a] = -1;
-            if (!has[q])
-                continue;
-            int lo0, hi0, lo1, hi1;
-            axis_window(mn[q][a], len[a], ks[a], g.neighbourhood, lo0, hi0);
-            axis_window(mx[q][a], len[a], ks[a], g.neighbourhood, lo1, hi1);
-            ulo[a] = min(ulo[a], lo0);
-            uhi[a] = max(uhi[a], hi1);
-            ilo[q][a] = lo1;      // bounds are monotone: the largest lo and the smallest hi
-            ihi[q][a] = hi0;
-        }
-    }
-    uint32_t *out = tlist + static_cast<size_t>(qp) * n_kt;
-    int n = 0;
-    for (int j = 0; j < n_kt; ++j) {
-        // does any of the tile's keys lie in the union box / in each intersection box?
-        bool any = false, all0 = true, all1 = true;
-        for (int e = lane; e < 128; e += 32) {
-            const int i = j * 128 + e;
-            if (i >= S)
-                continue;
-            int c[3];
-            grid_pos(g, i, c[0], c[1], c[2]);
-            bool in_u = true, in0 = true, in1 = true;
-#pragma unroll
-            for (int a = 0; a < 3; ++a) {
-                in_u &= c[a] >= ulo[a] && c[a] <= uhi[a];
-                in0 &= c[a] >= ilo[0][a] && c[a] <= ihi[0][a];
-                in1 &= c[a] >= ilo[1][a] && c[a] <= ihi[1][a];
-            }
-            any |= in_u;
-            all0 &= in0;
-            all1 &= in1;
-        }
-        any = __any_sync(0xFFFFFFFFu, any);
-        all0 = __all_sync(0xFFFFFFFFu, all0) && has[0];
-        all1 = __all_sync(0xFFFFFFFFu, all1) && has[1];
-        if (any) {
-            if (lane == 0)
-                out[n] = static_cast<uint32_t>(j) | (all0 ? 0u : 1u << SEG_MASK_SHIFT) |
-                         (all1 ? 0u : 1u << (SEG_MASK_SHIFT + 1));
-            ++n;
-        }
-    }
-    if (lane == 0)
-        tcount[qp] = n;
+    WinUnit u;
+    const int jw = qp % g.nuw;
+    const int r = qp / g.nuw;
+    const int jh = r % g.nuh;
+    const int jt = r / g.nuh;
+    u.t0 = jt << (g.qlt + 1);
+    u.h0 = jh << g.qlh;
+    u.w0 = jw << g.qlw;
+    int hi;
+    axis_union(u.t0, u.t0 + (2 << g.qlt) - 1, g.F, g.kt, g.neighbourhood, u.ut, hi);
+    u.nbt = (hi - u.ut + (1 << g.klt)) >> g.klt;
+    axis_union(u.h0, u.h0 + (1 << g.qlh) - 1, g.Hp, g.kh, g.neighbourhood, u.uh, hi);
+    u.nbh = (hi - u.uh + (1 << g.klh)) >> g.klh;
+    axis_union(u.w0, u.w0 + (1 << g.qlw) - 1, g.Wp, g.kw, g.neighbourhood, u.uw, hi);
+    u.nbw = (hi - u.uw + (1 << g.klw)) >> g.klw;
+    return u;
+}
+
+// Origin of key box r of a unit.
+__device__ __forceinline__ void win_box(const WinGrid &g, const WinUnit &u, int r, int &t, int &h, int &w)
+{
+    const int iw = r % u.nbw;
+    const int q = r / u.nbw;
+    const int ih = q % u.nbh;
+    const int it = q / u.nbh;
+    t = u.ut + (it << g.klt);
+    h = u.uh + (ih << g.klh);
+    w = u.uw + (iw << g.klw);
 }
 
 // Bits [lo, hi] (0 <= lo <= hi < 128) set in the 128-bit mask m.
@@ -169,46 +114,66 @@ __device__ __forceinline__ void set_bit_range(uint32_t (&m)[4], int lo, int hi)
     }
 }
 
-// The window of query token q, one axis per word: lo in the low 16 bits, hi in
-// the high 16 (grid sides below 65536).
-__device__ __forceinline__ void packed_window(const WinGrid &g, int q, uint32_t &tw, uint32_t &hw, uint32_t &ww)
+// Bits [lo, hi] of a 32-bit word (0 <= lo <= hi < 32).
+__device__ __forceinline__ uint32_t bit_range32(int lo, int hi)
 {
-    int qt, qh, qw, lo, hi;
-    grid_pos(g, q, qt, qh, qw);
-    axis_window(qt, g.F, g.kt, g.neighbourhood, lo, hi);
+    const int n = hi - lo + 1;
+    return (n == 32 ? 0xFFFFFFFFu : ((1u << n) - 1u)) << lo;
+}
+
+// A g-bit pattern (g a power of two, 1..32) repeated across a 32-bit word.
+__device__ __forceinline__ uint32_t repeat32(uint32_t pattern, int lg)
+{
+#pragma unroll
+    for (int s = 0; s < 5; ++s)
+        if (s >= lg)
+            pattern |= pattern << (1 << s);
+    return pattern;
+}
+
+// The window of a query at grid position (t, h, w), one axis per word: lo in
+// the low 16 bits, hi in the high 16 (grid sides below 65536).  A position
+// outside the grid (a ragged brick's padding row) gets empty windows.
+__device__ __forceinline__ void packed_window(const WinGrid &g, int t, int h, int w, uint32_t &tw, uint32_t &hw,
+                                              uint32_t &ww)
+{
+    if (t >= g.F || h >= g.Hp || w >= g.Wp) {
+        tw = hw = ww = 1u;   // lo = 1 > hi = 0
+        return;
+    }
+    int lo, hi;
+    axis_window(t, g.F, g.kt, g.neighbourhood, lo, hi);
     tw = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
-    axis_window(qh, g.Hp, g.kh, g.neighbourhood, lo, hi);
+    axis_window(h, g.Hp, g.kh, g.neighbourhood, lo, hi);
     hw = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
-    axis_window(qw, g.Wp, g.kw, g.neighbourhood, lo, hi);
+    axis_window(w, g.Wp, g.kw, g.neighbourhood, lo, hi);
     ww = static_cast<uint32_t>(lo) | (static_cast<uint32_t>(hi) << 16);
 }
 
-// 128-bit mask of the keys of key tile kt inside a query's window (packed as
-// above), given the grid position (t, h, w) of the tile's first key: the
-// tile's keys run through (t, h) rows of the grid; per row, the keys whose w
-// lies inside the window form one range.
-__device__ __forceinline__ void window_mask(const WinGrid &g, int S, uint32_t tw, uint32_t hw, uint32_t ww, int kt,
-                                            int t, int h, int w, uint32_t (&m)[4])
+// 128-bit mask of the keys of the key box with origin (t, h, w) inside a
+// query's window (packed as above).  Key c of the box sits at
+// (t + c / (kbh kbw), h + (c / kbw) % kbh, w + c % kbw).  The (h, w) pattern of
+// one t-slice (kbh x kbw bits, at most 32) is the w-range repeated over the
+// slice's rows and cut to the h-range; the mask repeats it over the t-slices
+// and cuts it to the t-range.
+__device__ __forceinline__ void window_mask(const WinGrid &g, uint32_t tw, uint32_t hw, uint32_t ww, int t, int h,
+                                            int w, uint32_t (&m)[4])
 {
     m[0] = m[1] = m[2] = m[3] = 0u;
-    const int tlo = static_cast<int>(tw & 0xFFFFu), thi = static_cast<int>(tw >> 16);
-    const int hlo = static_cast<int>(hw & 0xFFFFu), hhi = static_cast<int>(hw >> 16);
-    const int wlo = static_cast<int>(ww & 0xFFFFu), whi = static_cast<int>(ww >> 16);
-    const int kn = min(128, S - kt * 128);
-    for (int c = 0; c < kn;) {
-        const int len = min(g.Wp - w, kn - c);
-        if (t >= tlo && t <= thi && h >= hlo && h <= hhi) {
-            const int a = max(w, wlo), b = min(w + len - 1, whi);
-            if (a <= b)
-                set_bit_range(m, c + (a - w), c + (b - w));
-        }
-        c += len;
-        w = 0;
-        if (++h == g.Hp) {
-            h = 0;
-            ++t;
-        }
-    }
+    const int kbt = 1 << g.klt, kbh = 1 << g.klh, kbw = 1 << g.klw;
+    const int tlo = max(static_cast<int>(tw & 0xFFFFu) - t, 0), thi = min(static_cast<int>(tw >> 16) - t, kbt - 1);
+    const int hlo = max(static_cast<int>(hw & 0xFFFFu) - h, 0), hhi = min(static_cast<int>(hw >> 16) - h, kbh - 1);
+    const int wlo = max(static_cast<int>(ww & 0xFFFFu) - w, 0), whi = min(static_cast<int>(ww >> 16) - w, kbw - 1);
+    if (tlo > thi || hlo > hhi || wlo > whi)
+        return;
+    const int lg_slice = g.klh + g.klw;                     // log2 of the bits of one t-slice
+    const uint32_t slice =
+        repeat32(bit_range32(wlo, whi), g.klw) & bit_range32(hlo << g.klw, ((hhi + 1) << g.klw) - 1);
+    const uint32_t word = repeat32(slice, lg_slice);
+    set_bit_range(m, tlo << lg_slice, ((thi + 1) << lg_slice) - 1);
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        m[i] &= word;
 }
 
 }  // namespace vdx
