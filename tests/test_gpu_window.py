@@ -43,6 +43,9 @@ CASES = [
     (1, 1, 64, (1, 1, 1), (1, 1, 1), True),        # a single token
     (1, 3, 128, (9, 17, 23), (5, 3, 7), True),     # every side ragged against bricks and boxes
     (1, 2, 128, (21, 30, 52), (11, 11, 11), True),  # small480's grid with the decoder's window
+    # 156 units: every persistent CTA takes one, four take a second
+    (1, 13, 128, (8, 16, 24), (5, 5, 5), True),
+    (1, 13, 64, (8, 16, 24), (7, 3, 5), False),
 ]
 
 
