@@ -123,11 +123,11 @@ int vdx_attn_fwd_segments(const void *q, const void *k, const void *v, void *out
  *   neighbourhood = 1: [lo, min(lo + k, L) - 1], lo = clamp(p - k/2, 0, max(L - k, 0))
  *                      (shifted inward at the border: always min(k, L) positions);
  *   neighbourhood = 0: [max(p - k/2, 0), min(p + k/2, L - 1)] (truncated).
- * Key tiles (128 keys) outside every window of a query-tile pair are skipped;
- * the rest compare positions element by element.  A small kernel builds the
- * key-tile lists first, on the same stream, in the library's per-stream
- * workspace (ceil(S/256) x ceil(S/128) x 4 bytes).  Grid sides up to 65535;
- * VDX_ERR_UNSUPPORTED beyond.
+ * Query tiles are 3-D bricks of 128 tokens and key tiles 3-D boxes of 128
+ * tokens laid over the union of each unit's windows (shapes chosen per grid
+ * by the library); keys outside every window of a unit are never visited,
+ * and the rest compare positions element by element.  One kernel launch, no
+ * workspace.  Grid sides up to 65535; VDX_ERR_UNSUPPORTED beyond.
  */
 int vdx_attn_fwd_win3d(const void *q, const void *k, const void *v, void *out, float *lse,
                        int B, int H, int F, int Hp, int Wp, int D, int kt, int kh, int kw,
