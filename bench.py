@@ -203,12 +203,18 @@ def run_ours(args):
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with ClockSampler(local, clocks_log) as clk:
         barrier()
+        # one event between consecutive calls (recording an event launches
+        # no work): the per-call times below; the total spans them all
+        marks = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
         start.record(stream)
-        for _ in range(args.steps):
+        marks[0].record(stream)
+        for i in range(args.steps):
             step()
+            marks[i + 1].record(stream)
         end.record(stream)
         barrier()
     ms_total = max_over_ranks(start.elapsed_time(end), world, dev)
+    per_call = [marks[i].elapsed_time(marks[i + 1]) for i in range(args.steps)]
     st = binding.check_device_error(dev)
     if st != binding.VDX_OK:
         raise RuntimeError(binding.status_string(st))
@@ -295,6 +301,8 @@ def run_ours(args):
     line = {
         "metric": METRIC, "value": round(tflops, 2), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+        "ms_per_call": {"median": round(statistics.median(per_call), 4), "min": round(min(per_call), 4),
+                        "max": round(max(per_call), 4), "note": "rank 0, events between consecutive calls"},
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded N(0,1) bf16 tensors shaped like the workload; no dataset)",
         "config": {"workload": wl.name, "description": wl.description, "B": wl.B, "H": wl.H,
@@ -406,8 +414,10 @@ class OracleTimer:
     def run(self):
         dt = self._time(self.n)
         flops = self.flops_per_row * self.n * self.bh
+        full = self.flops_per_row * self.wl.Sq * self.bh   # the whole call's FLOP
         return {"value": round(flops / dt / 1e12, 6), "unit": UNIT, "cores": self.cores, "kind": "oracle",
                 "seconds": round(dt, 3),
+                "full_call_seconds_extrapolated": round(dt * full / flops, 1),
                 "sample": f"{self.n} seeded query rows per (b,h) x {self.bh} (b,h) pairs of workload "
                           f"{self.wl.name} ({flops:.3e} FLOP in fp64, OpenMP)"}
 
