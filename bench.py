@@ -288,7 +288,7 @@ def run_ours(args):
     # ---- oracle on the host cores (rank 0, N = 1 only)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = time_oracle(w, target_s=args.cpu_seconds)
+        cpu = time_oracle(w, target_s=args.cpu_seconds, gpu=(out, lse))
 
     if world > 1:
         dist.destroy_process_group()
@@ -396,12 +396,14 @@ class OracleTimer:
                          for _ in range(self.bh)]).astype(np.int32)
         t0 = time.perf_counter()
         if self.wl.window is not None:
-            self.orc.attn_fwd_win3d(*self.bits, self.wl.scale, self.wl.latent, self.wl.window[0],
-                                    self.wl.window[1], rows=rows)
+            res = self.orc.attn_fwd_win3d(*self.bits, self.wl.scale, self.wl.latent, self.wl.window[0],
+                                          self.wl.window[1], rows=rows)
         else:
-            self.orc.attn_fwd(*self.bits, self.wl.scale, kv_lens=self.w["kv_lens"], rows=rows,
-                              q_seg=self.w["q_seg"], kv_seg=self.w["kv_seg"])
-        return time.perf_counter() - t0
+            res = self.orc.attn_fwd(*self.bits, self.wl.scale, kv_lens=self.w["kv_lens"], rows=rows,
+                                    q_seg=self.w["q_seg"], kv_seg=self.w["kv_seg"])
+        dt = time.perf_counter() - t0
+        self.last = (rows, res)
+        return dt
 
     def calibrate(self, target_s):
         n, dt = 1, self._time(1)
@@ -422,10 +424,37 @@ class OracleTimer:
                           f"{self.wl.name} ({flops:.3e} FLOP in fp64, OpenMP)"}
 
 
-def time_oracle(w, target_s=15.0):
+def sample_parity(rows, ref, out, lse):
+    """The timed oracle sample against the GPU's output of the same call at
+    the same rows: max and mean |O| error, max relative LSE error (the
+    tolerances of the parity tests are 2e-2, 2e-3 and 1e-3)."""
+    import torch
+    o_ref, lse_ref = ref
+    B, H, Sq, D = out.shape
+    idx = torch.from_numpy(rows.astype(np.int64)).to(out.device).view(B, H, -1)
+    o = torch.gather(out, 2, idx.unsqueeze(-1).expand(-1, -1, -1, D)).float().double().cpu().numpy()
+    ls = torch.gather(lse, 2, idx).double().cpu().numpy()
+    err = np.abs(o - o_ref)
+    fin = np.isfinite(lse_ref)
+    rel = np.abs(ls[fin] - lse_ref[fin]) / np.maximum(1.0, np.abs(lse_ref[fin]))
+    return {"o_max_abs": float(f"{err.max():.3e}"), "o_mean_abs": float(f"{err.mean():.3e}"),
+            "lse_max_rel": float(f"{rel.max():.3e}") if rel.size else 0.0,
+            "lse_neg_inf_pattern_equal": bool(np.array_equal(np.isneginf(ls), ~fin)),
+            "rows": f"the timed sample's {rows.shape[1]} rows per (b,h)"}
+
+
+def time_oracle(w, target_s=15.0, gpu=None):
+    """The cpu_baseline record; with gpu = (out, lse) of the timed calls, the
+    sample's rows also serve as a parity spot check of that output."""
     t = OracleTimer(w)
     t.calibrate(target_s)
-    return t.run()
+    rec = t.run()
+    if gpu is not None:
+        if w["workload"].rope is not None:
+            rec["parity_on_sample"] = "not compared: this sample times the attention without the rotation"
+        else:
+            rec["parity_on_sample"] = sample_parity(*t.last, *gpu)
+    return rec
 
 
 def run_reference(args):
