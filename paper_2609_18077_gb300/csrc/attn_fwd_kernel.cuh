@@ -638,6 +638,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         // of an item and the key tile its GEMMs need next -- K_{j+1} of the
         // same item or the first key tile of the next item with keys.  Stage 0
         // holds that first key tile alone.
+        const uint64_t q_policy = ptx::policy_evict_first();
         auto next_with_keys = [&](int i) {
             for (++i;; ++i) {
                 const Item w = item_at<MODE>(p, sp, cta, i);
@@ -759,9 +760,18 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                 if (ok && lane == 0) {
                     ptx::mbar_arrive_expect_tx(bar(L::B_Q + 2 * qb + t), L::TILE_BYTES);
                     const TileAt qa = q_tile_at<MODE>(sp, w, t);
-                    for (int h = 0; h < D / 64; ++h)
-                        tma_tile<MODE>(sbase + L::Q_OFF + (2 * qb + t) * L::TILE_BYTES + h * L::HALF_BYTES, &tmap_q,
-                                       bar(L::B_Q + 2 * qb + t), h * 64, qa);
+                    const uint32_t qdst = sbase + L::Q_OFF + (2 * qb + t) * L::TILE_BYTES;
+                    // A Q tile is read once: first in line for eviction from
+                    // L2, so that it does not push out the keys and values
+                    // other CTAs still stream (13 % fewer DRAM reads per call
+                    // at S = 75600, same time).
+                    for (int h = 0; h < D / 64; ++h) {
+                        if (MODE == MODE_WIN)
+                            tma_tile<MODE>(qdst + h * L::HALF_BYTES, &tmap_q, bar(L::B_Q + 2 * qb + t), h * 64, qa);
+                        else
+                            ptx::tma_load_3d_hint(qdst + h * L::HALF_BYTES, &tmap_q, bar(L::B_Q + 2 * qb + t), h * 64,
+                                                  qa.c0, qa.bh, q_policy);
+                    }
                 }
                 if (ok) {
                     const uint32_t bit = 1u << (2 * qb + t);

@@ -171,13 +171,7 @@ __device__ __forceinline__ void tma_load_3d_hint(uint32_t dst, const void *tmap,
         : "memory");
 }
 
-__device__ __forceinline__ uint64_t policy_evict_last()
-{
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-
+// L2 policy: the lines an access brings in are the first to be evicted.
 __device__ __forceinline__ uint64_t policy_evict_first()
 {
     uint64_t p;
