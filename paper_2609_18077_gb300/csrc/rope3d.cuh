@@ -15,7 +15,7 @@
 // Memory-bound elementwise work (one read and one write of x): a thread owns
 // one pair (or, interleaved with D a multiple of 8, four consecutive pairs =
 // 16 bytes) of one token, computes the angles once and applies them to the
-// token's row in every (b, h), four rows in flight at a time, so a block
+// token's row in every (b, h), six rows in flight at a time, so a block
 // reads whole rows (consecutive tokens are consecutive rows) and the sine and
 // cosine cost is shared by the B*H rows.
 #pragma once
@@ -117,7 +117,7 @@ __device__ __forceinline__ uint32_t rotate_pair(uint32_t word, float c, float sn
     return *reinterpret_cast<const uint32_t *>(&o);
 }
 
-constexpr int ROPE_ROWS = 4;   // (b, h) rows loaded before any is stored
+constexpr int ROPE_ROWS = 6;   // (b, h) rows loaded before any is stored
 
 // Interleaved pairing, D a multiple of 8: one token's 16-byte chunk q4 (four
 // consecutive pairs) in every (b, h) row.
