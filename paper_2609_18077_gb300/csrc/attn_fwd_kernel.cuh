@@ -71,6 +71,7 @@
 
 #include <cuda.h>
 #include <cuda_bf16.h>
+#include <climits>
 #include <cstdint>
 
 #include "segment_tiles.cuh"
@@ -941,6 +942,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
         const uint32_t o_addr = lane_addr + 256 + 128 * t;
         const float sl2 = p.scale_log2;
         const bool neg_scale = sl2 < 0.f;
+        // MODE_WIN: the combs of window_mask and its cache of t-range words
+        const uint32_t comb_w = MODE == MODE_WIN ? repeat32(1u, sp.win.klw) : 0u;
+        const uint32_t comb_s = MODE == MODE_WIN ? repeat32(1u, sp.win.klh + sp.win.klw) : 0u;
+        int win_tc = INT_MIN;
+        uint32_t win_tm[4] = {0u, 0u, 0u, 0u};
         int g = 1;      // stage of the current item's (V_j0, next K)
         int sc = 0;     // S phases consumed
         int iq = 0;     // items with keys so far
@@ -948,6 +954,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
 
         for (int i = 0; ok; ++i) {
             const Item w = item_at<MODE>(p, sp, cta, i);
+            win_tc = INT_MIN;   // the row's window changes with the unit
             if (!w.ok)
                 break;
             // This row's query: its token index q_row (stores and LSE) and, in
@@ -996,7 +1003,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1)
                         reinterpret_cast<volatile uint32_t *>(sm + L::ENTRY_OFF) + 4 * (gj % L::NSTAGE);
                     const uint32_t th = slot[1];
                     window_mask(sp.win, win_t, win_h, win_w, static_cast<int>(th & 0xFFFFu),
-                                static_cast<int>(th >> 16), static_cast<int>(slot[2]), wmask);
+                                static_cast<int>(th >> 16), static_cast<int>(slot[2]), comb_w, comb_s, win_tc, win_tm,
+                                wmask);
                 }
                 uint32_t s[4][32];
 #pragma unroll

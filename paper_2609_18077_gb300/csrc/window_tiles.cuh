@@ -155,25 +155,32 @@ __device__ __forceinline__ void packed_window(const WinGrid &g, int t, int h, in
 // (t + c / (kbh kbw), h + (c / kbw) % kbh, w + c % kbw).  The (h, w) pattern of
 // one t-slice (kbh x kbw bits, at most 32) is the w-range repeated over the
 // slice's rows and cut to the h-range; the mask repeats it over the t-slices
-// and cuts it to the t-range.
+// and cuts it to the t-range.  A repetition is one multiplication: a pattern
+// narrower than its group times a comb (a 1 at the start of every group; no
+// two copies overlap, so there is no carry).  comb_w has a 1 every kbw bits,
+// comb_s every kbh kbw bits.  The t-range words depend only on the row's
+// window and the box's t; they are kept in tm for the last t seen (tc), which
+// the caller resets whenever the row's window changes.
 __device__ __forceinline__ void window_mask(const WinGrid &g, uint32_t tw, uint32_t hw, uint32_t ww, int t, int h,
-                                            int w, uint32_t (&m)[4])
+                                            int w, uint32_t comb_w, uint32_t comb_s, int &tc, uint32_t (&tm)[4],
+                                            uint32_t (&m)[4])
 {
-    m[0] = m[1] = m[2] = m[3] = 0u;
-    const int kbt = 1 << g.klt, kbh = 1 << g.klh, kbw = 1 << g.klw;
-    const int tlo = max(static_cast<int>(tw & 0xFFFFu) - t, 0), thi = min(static_cast<int>(tw >> 16) - t, kbt - 1);
-    const int hlo = max(static_cast<int>(hw & 0xFFFFu) - h, 0), hhi = min(static_cast<int>(hw >> 16) - h, kbh - 1);
-    const int wlo = max(static_cast<int>(ww & 0xFFFFu) - w, 0), whi = min(static_cast<int>(ww >> 16) - w, kbw - 1);
-    if (tlo > thi || hlo > hhi || wlo > whi)
-        return;
-    const int lg_slice = g.klh + g.klw;                     // log2 of the bits of one t-slice
-    const uint32_t slice =
-        repeat32(bit_range32(wlo, whi), g.klw) & bit_range32(hlo << g.klw, ((hhi + 1) << g.klw) - 1);
-    const uint32_t word = repeat32(slice, lg_slice);
-    set_bit_range(m, tlo << lg_slice, ((thi + 1) << lg_slice) - 1);
+    if (t != tc) {
+        tc = t;
+        tm[0] = tm[1] = tm[2] = tm[3] = 0u;
+        const int tlo = max(static_cast<int>(tw & 0xFFFFu) - t, 0);
+        const int thi = min(static_cast<int>(tw >> 16) - t, (1 << g.klt) - 1);
+        if (tlo <= thi)
+            set_bit_range(tm, tlo << (g.klh + g.klw), ((thi + 1) << (g.klh + g.klw)) - 1);
+    }
+    const int hlo = max(static_cast<int>(hw & 0xFFFFu) - h, 0), hhi = min(static_cast<int>(hw >> 16) - h, (1 << g.klh) - 1);
+    const int wlo = max(static_cast<int>(ww & 0xFFFFu) - w, 0), whi = min(static_cast<int>(ww >> 16) - w, (1 << g.klw) - 1);
+    uint32_t word = 0u;
+    if (hlo <= hhi && wlo <= whi)
+        word = ((bit_range32(wlo, whi) * comb_w) & bit_range32(hlo << g.klw, ((hhi + 1) << g.klw) - 1)) * comb_s;
 #pragma unroll
     for (int i = 0; i < 4; ++i)
-        m[i] &= word;
+        m[i] = tm[i] & word;
 }
 
 }  // namespace vdx
