@@ -58,6 +58,13 @@ MUTANTS = {
     "win_truncated_radius": [("*hi = p + k / 2 < L - 1 ? p + k / 2 : L - 1;", "*hi = p + k / 2 - 1 < L - 1 ? p + k / 2 - 1 : L - 1;")],
     "win_key_index_axes": [("idx[n++] = (tt * Hp + hh) * Wp + ww;", "idx[n++] = (tt * Wp + hh) * Hp + ww;")],
     "win_w_axis_uses_h_size": [("axis_window(pw, Wp, kw,", "axis_window(pw, Wp, kh,")],
+    "win_neighbourhood_one_past": [("*hi = start + k - 1 < L - 1 ? start + k - 1 : L - 1;",
+                                    "*hi = start + k < L - 1 ? start + k : L - 1;")],
+    "win_truncated_lo_clamped_to_one": [("*lo = p - k / 2 > 0 ? p - k / 2 : 0;", "*lo = p - k / 2 > 0 ? p - k / 2 : 1;")],
+    "win_border_rule_inverted": [("    if (neighbourhood) {\n        int start", "    if (!neighbourhood) {\n        int start")],
+    "rope_passthrough_zeroed": [("            yr[d] = bf16_to_f64(xr[d]);", "            yr[d] = 0.0;")],
+    "rope_turns_tokens_after_grid": [("if (g < 0 || g >= grid)", "if (g < 0)")],
+    "empty_row_lse_zero": [("*lse = -INFINITY;", "*lse = 0.0;")],
 }
 
 CHILD = r"""
