@@ -30,6 +30,7 @@ namespace {
 constexpr int kVersion = 1 * 10000 + 0 * 100 + 0;
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s per in-kernel wait
 constexpr int kMaxDevices = 64;
+constexpr int kMinPartTiles = 8;   // key tiles a part of a cut single-round call holds at least
 
 using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                    const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
@@ -408,17 +409,29 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     // Persistent grid: one CTA per multiprocessor (one fits per SM), each
     // taking units blockIdx.x, blockIdx.x + grid, ... so that the CTAs
     // running at any moment work on neighbouring units of the same heads.
-    const int G = p.units < sms ? p.units : sms;
-    const dim3 grid(static_cast<unsigned>(G));
+    int G = p.units < sms ? p.units : sms;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
 
     // Short last round: when at most half the CTAs would get a unit in it,
     // cut each of those units along the keys into parts, one per CTA, and
-    // merge the parts (dense problems; varlen units vary in length).
+    // merge the parts (dense problems; varlen units vary in length).  A
+    // dense call of at most half as many units as multiprocessors has only
+    // such a round: its units are cut the same way, onto units x parts CTAs,
+    // each part at least kMinPartTiles key tiles (shorter parts measured
+    // slower than no cut: the merge outweighs them).
     const int n_kv = (Skv + vdx::BN - 1) / vdx::BN;
-    const int full_rounds = p.units / G;
-    const int tail = p.units - full_rounds * G;
-    int parts = (rule.mode == vdx::MODE_DENSE && full_rounds >= 1 && tail > 0) ? G / tail : 0;
+    int full_rounds = p.units / G;
+    int tail = p.units - full_rounds * G;
+    int parts = 0;
+    if (rule.mode == vdx::MODE_DENSE && p.units > 0 && 2 * p.units <= sms) {
+        full_rounds = 0;
+        tail = p.units;
+        parts = sms / tail;
+        if (parts > n_kv / kMinPartTiles)
+            parts = n_kv / kMinPartTiles;
+    } else if (rule.mode == vdx::MODE_DENSE && full_rounds >= 1 && tail > 0) {
+        parts = G / tail;
+    }
     if (parts > n_kv)
         parts = n_kv;
     if (parts >= 2) {
@@ -440,6 +453,8 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
         p.split_parts = parts;
         p.full_rounds = full_rounds;
         p.tail_units = tail;
+        if (full_rounds == 0)
+            G = tail * parts;
         p.ws_o = static_cast<float *>(ws);
         p.ws_stats = reinterpret_cast<float *>(static_cast<char *>(ws) + sl.o_bytes);
         p.ws_count = reinterpret_cast<int *>(static_cast<char *>(ws) + sl.o_bytes + sl.st_bytes);
@@ -486,6 +501,7 @@ int attn_launch(const void *q, const void *k, const void *v, void *out, float *l
     using vdx::MODE_SEG;
     using vdx::MODE_VARLEN;
     using vdx::MODE_WIN;
+    const dim3 grid(static_cast<unsigned>(G));
     cudaError_t e;
     if (D == 128) {
         e = varlen ? launch<128, MODE_VARLEN, 1, 2>(grid, mq, mk, mv, mo, p, sp, s)
@@ -653,6 +669,12 @@ std::vector<HostChunk> make_chunks(long long r, int B, int H, bool per_sample)
 // dense split applies (attn_launch's rule).
 double launch_rounds(long long units, int sms, int n_kv, bool dense)
 {
+    if (dense && units > 0 && 2 * units <= sms) {   // a single round cut along the keys
+        long long parts = sms / units;
+        if (parts > n_kv / kMinPartTiles)
+            parts = n_kv / kMinPartTiles;
+        return parts >= 2 ? 1.0 / static_cast<double>(parts) : 1.0;
+    }
     const long long G = units < sms ? units : sms;
     const long long full = units / G, tail = units - full * G;
     if (tail == 0)

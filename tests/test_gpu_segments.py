@@ -97,7 +97,8 @@ def test_segments(name):
 @pytest.mark.parametrize("D", [64, 128])
 def test_one_segment_is_the_dense_kernel(D):
     """A single id everywhere visits every tile unmasked: bit-identical to vdx_attn_fwd
-    (the sizes keep the dense call on whole units, without the split tail)."""
+    (the sizes keep the dense call on whole units: 24 units with 7 key tiles,
+    too few for a cut of at least 8 tiles a part)."""
     B, H, S = 2, 3, 777
     q, k, v = workloads.random_qkv(B, H, S, S, D, seed=61 + D, logit_gain=1.5)
     seg = np.full((B, S), 42, np.int32)
