@@ -28,7 +28,9 @@
  *   - All tensor pointers are DEVICE pointers owned by the caller; the
  *     library never frees or keeps them after the call returns.
  *   - Memory: when the last round of work units would leave most
- *     multiprocessors idle (dense calls only), the library splits those units
+ *     multiprocessors idle (dense calls only; a call of at most half as many
+ *     units as multiprocessors is all such a round, cut into parts of at
+ *     least 8 key tiles), the library splits those units
  *     along the keys and merges the parts through a device scratch of at most
  *     (multiprocessors x 2 x 128 x (D + 4)) fp32 values plus counters -- about
  *     20.6 MB on a 152-SM GB300.  It is allocated at that bound by the first
